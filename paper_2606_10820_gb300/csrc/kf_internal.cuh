@@ -1,0 +1,213 @@
+// Internal declarations shared by the library's CUDA translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/kforcing.h"
+
+namespace kf {
+
+constexpr int kMaxHeadDim = 64;   // head_dim is 32 or 64
+constexpr int kPage = 16;
+constexpr int kChunk = 32;          // vocab ids per LM-head record
+constexpr int kMaxGroupRows = 16;   // query rows per attention CTA
+
+// device error bits (ORed into ctx->d_err)
+constexpr int kErrBadToken = 1;
+constexpr int kErrBadPage = 2;
+constexpr int kErrTimeout = 4;
+constexpr int kErrBadRow = 8;
+
+__host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+__host__ __device__ inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
+
+// storage <-> fp32
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float x) {
+  return __float2bfloat16_rn(x);
+}
+
+__device__ __forceinline__ float gelu_tanh(float x) {
+  const float c = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * x * (1.0f + tanhf(c * (x + 0.044715f * x * x * x)));
+}
+
+// ---------------------------------------------------------------- GEMM epilogues
+// Every GEMM computes D[M][N] = A[M][K] . W[N][K]^T with fp32 accumulation and
+// hands each thread runs of 32 consecutive columns of one row to epi_run32.
+enum EpiKind : int {
+  EPI_STORE = 0,      // out[row][col] = D            (storage type TA)
+  EPI_BIAS_GELU = 1,  // out[row][col] = gelu(D + bias[col])
+  EPI_RESID = 2,      // x[row][col] += D             (fp32 residual stream)
+  EPI_NOISE_OUT = 3,  // x[map[row]][col] = D + bias[col] (+ pos_emb[pos][col])
+  EPI_HEAD = 4,       // per (row, 32-id chunk): max, sum exp(l - max), argmax of l = D/tau
+  EPI_LOGITS = 5,     // outf[row][col] = D / tau     (fp32, col < n_valid)
+  EPI_STORE_F32 = 6,  // outf[row][col] = D
+};
+
+struct HeadRec {   // one record per (head row, chunk of 32 vocab ids)
+  float m;         // max of l over the chunk
+  float s;         // sum over the chunk of exp(l - m), ascending id order
+  int a;           // lowest id attaining m
+  int pad;
+};
+
+struct Epi {
+  int kind = EPI_STORE;
+  void* out = nullptr;          // TA
+  float* outf = nullptr;        // fp32 outputs
+  int ldo = 0;
+  const float* bias = nullptr;
+  float* x = nullptr;           // residual stream
+  int ldx = 0;
+  const int32_t* row_map = nullptr;
+  const int32_t* row_pos = nullptr;
+  const float* pos_emb = nullptr;
+  float inv_tau = 1.0f;
+  int n_valid = 0;
+  HeadRec* rec = nullptr;
+  int nchunk = 0;
+};
+
+template <typename TA>
+__device__ __forceinline__ void epi_run32(const Epi& e, int row, int col0, const float* v, int N) {
+  switch (e.kind) {
+    case EPI_STORE: {
+      TA* o = reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < N) o[j] = from_f<TA>(v[j]);
+      break;
+    }
+    case EPI_STORE_F32: {
+      float* o = e.outf + (size_t)row * e.ldo + col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < N) o[j] = v[j];
+      break;
+    }
+    case EPI_BIAS_GELU: {
+      TA* o = reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < N) o[j] = from_f<TA>(gelu_tanh(v[j] + (e.bias ? e.bias[col0 + j] : 0.f)));
+      break;
+    }
+    case EPI_RESID: {
+      float* o = e.x + (size_t)row * e.ldx + col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < N) o[j] += v[j];
+      break;
+    }
+    case EPI_NOISE_OUT: {
+      int xr = e.row_map[row];
+      float* o = e.x + (size_t)xr * e.ldx + col0;
+      const float* pe = e.pos_emb ? e.pos_emb + (size_t)e.row_pos[xr] * N + col0 : nullptr;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < N) o[j] = v[j] + (e.bias ? e.bias[col0 + j] : 0.f) + (pe ? pe[j] : 0.f);
+      break;
+    }
+    case EPI_HEAD: {
+      // col0 is a multiple of 32: one record for ids col0 .. col0+31 (< n_valid)
+      int nv = e.n_valid - col0;
+      if (nv <= 0) break;
+      if (nv > 32) nv = 32;
+      float m = -INFINITY;
+      int a = col0;
+      for (int j = 0; j < nv; ++j) {
+        float l = v[j] * e.inv_tau;
+        if (l > m) { m = l; a = col0 + j; }
+      }
+      float s = 0.f;
+      for (int j = 0; j < nv; ++j) s += expf(v[j] * e.inv_tau - m);
+      HeadRec r;
+      r.m = m; r.s = s; r.a = a; r.pad = 0;
+      e.rec[(size_t)row * e.nchunk + col0 / 32] = r;
+      break;
+    }
+    case EPI_LOGITS: {
+      float* o = e.outf + (size_t)row * e.ldo + col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (col0 + j < e.n_valid) o[j] = v[j] * e.inv_tau;
+      break;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- launches
+struct GemmDesc {
+  int M, N, K;
+  const void* A;   // [M][lda] storage TA
+  int lda;
+  const void* W;   // [N][ldw] storage TA
+  int ldw;
+  Epi epi;
+};
+
+// SIMT GEMM (any storage type; fp32 accumulation, k ascending per output)
+void launch_gemm_simt(bool bf16, const GemmDesc& g, cudaStream_t s);
+
+// tcgen05 GEMM (bf16 only).  Requires K % 64 == 0, 16-byte aligned rows,
+// A rows readable up to round_up(M,128), W rows up to round_up(N,BN).
+struct TcPlan;
+bool tc_gemm_supported(const GemmDesc& g);
+int launch_gemm_tc(const GemmDesc& g, void* workspace, size_t ws_bytes, int* counters,
+                   int n_counters, int* d_err, cudaStream_t s);
+
+struct AttnArgs {
+  const float* q;          // [R][H][hd] (rotated, unscaled)
+  const void* kv;          // pool [L][n_pages][2][H][16][hd]
+  int layer, n_pages, H, hd;
+  const int32_t* page_table;  // [max_batch][max_pages]
+  int max_pages;
+  const int32_t* row_seq;  // [R]
+  const int32_t* row_pos;  // [R]
+  const int4* groups;      // {b, row0, nrows, 0} or NULL (uniform: group g = seq g)
+  int uniform_rows;        // rows per sequence when groups == NULL
+  void* out;               // [R][H*hd] TA
+  float* part_o;           // [n_split][R][H][hd]
+  float2* part_ml;         // [n_split][R][H]
+  int R;
+  int n_split;
+  int keys_per_split;      // multiple of 64
+  int* d_err;
+};
+void launch_attention(bool bf16, const AttnArgs& a, int n_groups, cudaStream_t s);
+void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
+
+// elementwise / bookkeeping kernels
+void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
+                   int32_t* noise_map, int32_t* head_map, cudaStream_t s);
+void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
+                          const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
+                          int V, int d, float* x, int* d_err, cudaStream_t s);
+void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
+                         const float* pos_emb, const int32_t* row_pos, int V, int d, float* x,
+                         int* d_err, cudaStream_t s);
+void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
+                       float scale, int d, void* feat, cudaStream_t s);
+void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
+                    const float* g, float eps, void* out, cudaStream_t s);
+void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
+                        const int32_t* row_seq,
+                        const int32_t* row_pos, const float* cos_t, const float* sin_t, float* q,
+                        void* kv, int layer, int n_pages, const int32_t* page_table, int max_pages,
+                        int* d_err, cudaStream_t s);
+void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
+                        int d, const void* w_head, int V, float inv_tau, int map_kind,
+                        const float* noise, int32_t* tokens, cudaStream_t s);
+void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
+                   int32_t* d_len, cudaStream_t s);
+
+}  // namespace kf

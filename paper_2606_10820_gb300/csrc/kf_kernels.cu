@@ -1,0 +1,421 @@
+// Row bookkeeping, embeddings, noise features, RMSNorm, RoPE + KV append,
+// the LM head's noise -> token selection, and the step commit.
+#include <algorithm>
+
+#include "kf_internal.cuh"
+
+namespace kf {
+
+// ------------------------------------------------------------------ rows
+// Alg. 1 row layout per sequence b: P pending tokens at positions
+// c_b .. c_b+P-1, then k noise slots at c_b+P .. c_b+P+k-1.
+__global__ void k_rowmap(int B, int P, int k, const int32_t* __restrict__ len,
+                         int32_t* row_seq, int32_t* row_pos, int32_t* noise_map,
+                         int32_t* head_map) {
+  int r = blockIdx.x * blockDim.x + threadIdx.x;
+  int S = P + k;
+  if (r < B * S) {
+    int b = r / S, i = r - b * S;
+    row_seq[r] = b;
+    row_pos[r] = len[b] + i;
+  }
+  if (k > 0 && r < B * k) {
+    int b = r / k, j = r - b * k;
+    noise_map[r] = b * S + P + j;
+    head_map[r] = b * S + P + j;
+  }
+  if (k == 0 && r < B) head_map[r] = r * S + P - 1;
+}
+
+void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
+                   int32_t* noise_map, int32_t* head_map, cudaStream_t s) {
+  int n = B * (P + k);
+  k_rowmap<<<ceil_div(n, 128), 128, 0, s>>>(B, P, k, d_len, row_seq, row_pos, noise_map, head_map);
+}
+
+// ------------------------------------------------------------ embeddings
+template <typename TA>
+__device__ void embed_row(int r, int tok, int pos, const TA* __restrict__ emb,
+                          const float* __restrict__ pos_emb, int V, int d, float* x, int* d_err) {
+  float* o = x + (size_t)r * d;
+  if (tok < 0 || tok >= V) {
+    if (threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
+    for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = 0.f;
+    return;
+  }
+  const TA* e = emb + (size_t)tok * d;
+  const float* p = pos_emb ? pos_emb + (size_t)pos * d : nullptr;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = to_f(e[c]) + (p ? p[c] : 0.f);
+}
+
+template <typename TA>
+__global__ void k_embed_pending(int P, int k, const int32_t* __restrict__ pending, int pend_stride,
+                                const TA* __restrict__ emb, const float* __restrict__ pos_emb,
+                                const int32_t* __restrict__ row_pos, int V, int d, float* x,
+                                int* d_err) {
+  int b = blockIdx.x / P, i = blockIdx.x - b * P;
+  int r = b * (P + k) + i;
+  embed_row<TA>(r, pending[b * pend_stride + i], row_pos[r], emb, pos_emb, V, d, x, d_err);
+}
+
+template <typename TA>
+__global__ void k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
+                               const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
+                               int V, int d, float* x, int* d_err) {
+  int r = blockIdx.x;
+  embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, d_err);
+}
+
+void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
+                          const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
+                          int V, int d, float* x, int* d_err, cudaStream_t s) {
+  if (B * P == 0) return;
+  if (bf16)
+    k_embed_pending<__nv_bfloat16><<<B * P, 128, 0, s>>>(P, k, pending, pend_stride,
+        (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
+  else
+    k_embed_pending<float><<<B * P, 128, 0, s>>>(P, k, pending, pend_stride,
+        (const float*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
+}
+
+void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
+                         const float* pos_emb, const int32_t* row_pos, int V, int d, float* x,
+                         int* d_err, cudaStream_t s) {
+  if (R == 0) return;
+  if (bf16)
+    k_embed_tokens<__nv_bfloat16><<<R, 128, 0, s>>>(row_tok, (const __nv_bfloat16*)tok_emb,
+                                                    pos_emb, row_pos, V, d, x, d_err);
+  else
+    k_embed_tokens<float><<<R, 128, 0, s>>>(row_tok, (const float*)tok_emb, pos_emb, row_pos, V,
+                                            d, x, d_err);
+}
+
+// ------------------------------------------------------- noise features
+// Sinusoidal encoding of z and of tau (Table 4), summed; argument
+// scale * u * freq[t], freq[t] = exp(-ln(1e4) t / (d/2)); [cos | sin].
+// Angles are formed in fp64 so the feature is the fp32 rounding of the
+// exact value.
+template <typename TA>
+__global__ void k_noise_feat(int n, const float* __restrict__ noise, const double* __restrict__ freq,
+                             float tau, float scale, int d, TA* __restrict__ feat) {
+  int half = d / 2;
+  int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= n * half) return;
+  int r = idx / half, t = idx - r * half;
+  double f = freq[t];
+  double az = (double)scale * (double)noise[r] * f;
+  double at = (double)scale * (double)tau * f;
+  double sz, cz, st, ct;
+  sincos(az, &sz, &cz);
+  sincos(at, &st, &ct);
+  feat[(size_t)r * d + t] = from_f<TA>((float)(cz + ct));
+  feat[(size_t)r * d + half + t] = from_f<TA>((float)(sz + st));
+}
+
+void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
+                       float scale, int d, void* feat, cudaStream_t s) {
+  if (n == 0) return;
+  int tot = n * (d / 2);
+  if (bf16)
+    k_noise_feat<__nv_bfloat16><<<ceil_div(tot, 256), 256, 0, s>>>(n, noise, freq, tau, scale, d,
+                                                                   (__nv_bfloat16*)feat);
+  else
+    k_noise_feat<float><<<ceil_div(tot, 256), 256, 0, s>>>(n, noise, freq, tau, scale, d,
+                                                           (float*)feat);
+}
+
+// --------------------------------------------------------------- RMSNorm
+// out[r] = x[src] / sqrt(mean(x[src]^2) + eps) * g   (Table 4 pre-norm)
+template <typename TA>
+__global__ void k_rmsnorm(const int32_t* __restrict__ row_map, const float* __restrict__ x, int d,
+                          const float* __restrict__ g, float eps, TA* __restrict__ out) {
+  int r = blockIdx.x;
+  int src = row_map ? row_map[r] : r;
+  const float* xr = x + (size_t)src * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += xr[c] * xr[c];
+  __shared__ float red[32];
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  float inv = rsqrtf(red[0] / (float)d + eps);
+  TA* o = out + (size_t)r * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = from_f<TA>(xr[c] * inv * g[c]);
+}
+
+void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
+                    const float* g, float eps, void* out, cudaStream_t s) {
+  if (R == 0) return;
+  if (bf16)
+    k_rmsnorm<__nv_bfloat16><<<R, 128, 0, s>>>(row_map, x, d, g, eps, (__nv_bfloat16*)out);
+  else
+    k_rmsnorm<float><<<R, 128, 0, s>>>(row_map, x, d, g, eps, (float*)out);
+}
+
+// ------------------------------------------------------ RoPE + KV append
+// Rotate q and k of every row at its position (pairs (i, i+hd/2)), keep the
+// rotated q (fp32) for attention and write k, v of ALL rows (pending and
+// noise) into the paged cache.  Noise rows' entries sit at positions the
+// next step overwrites with committed tokens (Alg. 1 discards C_z).
+// KV pool layout: [layer][page][K|V][head][16 slots][hd].
+template <typename TA, int HD>
+__global__ void k_rope_append(const TA* __restrict__ qkv, int d, int H,
+                              const int32_t* __restrict__ row_seq, const int32_t* __restrict__ row_pos,
+                              const float* __restrict__ cos_t, const float* __restrict__ sin_t,
+                              float* __restrict__ q, TA* __restrict__ kv, int layer, int n_pages,
+                              const int32_t* __restrict__ page_table, int max_pages, int* d_err) {
+  constexpr int HALF = HD / 2;
+  int r = blockIdx.x;
+  int h = threadIdx.x / HALF, i = threadIdx.x % HALF;
+  if (h >= H) return;
+  int b = row_seq[r], pos = row_pos[r];
+  const TA* src = qkv + (size_t)r * 3 * d + h * HD;
+  float q1 = to_f(src[i]), q2 = to_f(src[i + HALF]);
+  float k1 = to_f(src[d + i]), k2 = to_f(src[d + i + HALF]);
+  float v1 = to_f(src[2 * d + i]), v2 = to_f(src[2 * d + i + HALF]);
+  if (cos_t) {
+    float c = cos_t[pos * HALF + i], sn = sin_t[pos * HALF + i];
+    float a1 = q1 * c - q2 * sn, a2 = q2 * c + q1 * sn;
+    q1 = a1; q2 = a2;
+    float b1 = k1 * c - k2 * sn, b2 = k2 * c + k1 * sn;
+    k1 = b1; k2 = b2;
+  }
+  float* qo = q + ((size_t)r * H + h) * HD;
+  qo[i] = q1;
+  qo[i + HALF] = q2;
+  int pi = pos / kPage;
+  int page = (pi < max_pages) ? page_table[b * max_pages + pi] : -1;
+  if (page < 0 || page >= n_pages) {
+    if (i == 0) atomicOr(d_err, kErrBadPage);
+    return;
+  }
+  size_t base = ((((size_t)layer * n_pages + page) * 2) * H + h) * (kPage * HD) +
+                (size_t)(pos % kPage) * HD;
+  size_t vofs = (size_t)H * kPage * HD;
+  kv[base + i] = from_f<TA>(k1);
+  kv[base + i + HALF] = from_f<TA>(k2);
+  kv[base + vofs + i] = from_f<TA>(v1);
+  kv[base + vofs + i + HALF] = from_f<TA>(v2);
+}
+
+template <int HD>
+static void rope_append_hd(bool bf16, int R, const void* qkv, int d, int H, const int32_t* row_seq,
+                           const int32_t* row_pos, const float* cos_t, const float* sin_t, float* q,
+                           void* kv, int layer, int n_pages, const int32_t* page_table,
+                           int max_pages, int* d_err, cudaStream_t s) {
+  int threads = H * (HD / 2);
+  if (bf16)
+    k_rope_append<__nv_bfloat16, HD><<<R, threads, 0, s>>>((const __nv_bfloat16*)qkv, d, H,
+        row_seq, row_pos, cos_t, sin_t, q, (__nv_bfloat16*)kv, layer, n_pages, page_table,
+        max_pages, d_err);
+  else
+    k_rope_append<float, HD><<<R, threads, 0, s>>>((const float*)qkv, d, H, row_seq, row_pos,
+        cos_t, sin_t, q, (float*)kv, layer, n_pages, page_table, max_pages, d_err);
+}
+
+void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
+                        const int32_t* row_seq, const int32_t* row_pos, const float* cos_t,
+                        const float* sin_t, float* q, void* kv, int layer, int n_pages,
+                        const int32_t* page_table, int max_pages, int* d_err, cudaStream_t s) {
+  if (R == 0) return;
+  if (hd == 64)
+    rope_append_hd<64>(bf16, R, qkv, d, H, row_seq, row_pos, cos_t, sin_t, q, kv, layer, n_pages,
+                       page_table, max_pages, d_err, s);
+  else
+    rope_append_hd<32>(bf16, R, qkv, d, H, row_seq, row_pos, cos_t, sin_t, q, kv, layer, n_pages,
+                       page_table, max_pages, d_err, s);
+}
+
+// ------------------------------------------------- noise -> token select
+// Combines the per-chunk records of one head row (l = logits / tau):
+//   M = max_c m_c,  S = sum_c s_c exp(m_c - M)        (chunks in id order)
+// ICDF (Eq. 1, App. B strict '>'): T = z S; the first chunk c* whose running
+// sum exceeds T; its 32 logits are recomputed and the first id whose running
+// sum (from the chunk start, T' = T - sum before c*) exceeds T' is the token.
+// If rounding leaves no crossing, the largest id with exp(l - M) > 0 wins.
+// ARGMAX: the lowest id attaining M.
+constexpr int kSelThreads = 256;
+
+template <typename TA>
+__global__ void __launch_bounds__(kSelThreads)
+k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
+              const TA* __restrict__ w_head, int V, float inv_tau, int map_kind,
+              const float* __restrict__ noise, int32_t* __restrict__ tokens) {
+  const int row = blockIdx.x;
+  const HeadRec* rec = rec_all + (size_t)row * nchunk;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  __shared__ float s_red[kSelThreads / 32];
+  __shared__ int s_redi[kSelThreads / 32];
+  __shared__ float s_part[kSelThreads];
+  __shared__ float s_M, s_T;
+  __shared__ int s_chunk;
+  __shared__ float s_before;
+
+  // contiguous chunk range per thread keeps id order inside each partial sum
+  const int per = ceil_div(nchunk, kSelThreads);
+  const int c0 = min(nchunk, t * per), c1 = min(nchunk, c0 + per);
+
+  // 1) M and (for argmax) the lowest id attaining it
+  float m = -INFINITY;
+  int am = 0x7fffffff;
+  for (int c = c0; c < c1; ++c) {
+    HeadRec r = rec[c];
+    if (r.m > m) { m = r.m; am = r.a; }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    int a2 = __shfl_xor_sync(0xffffffffu, am, o);
+    if (m2 > m || (m2 == m && a2 < am)) { m = m2; am = a2; }
+  }
+  if (lane == 0) { s_red[warp] = m; s_redi[warp] = am; }
+  __syncthreads();
+  if (t == 0) {
+    float M = s_red[0];
+    int A = s_redi[0];
+    for (int w = 1; w < kSelThreads / 32; ++w)
+      if (s_red[w] > M || (s_red[w] == M && s_redi[w] < A)) { M = s_red[w]; A = s_redi[w]; }
+    s_M = M;
+    s_redi[0] = A;
+  }
+  __syncthreads();
+  if (map_kind == KF_MAP_ARGMAX) {
+    if (t == 0) tokens[row] = s_redi[0];
+    return;
+  }
+  const float M = s_M;
+
+  // 2) per-thread partial sums, then an ordered scan over threads
+  float part = 0.f;
+  for (int c = c0; c < c1; ++c) {
+    HeadRec r = rec[c];
+    part += r.s * expf(r.m - M);
+  }
+  s_part[t] = part;
+  __syncthreads();
+  if (t == 0) {
+    float S = 0.f;
+    for (int i = 0; i < kSelThreads; ++i) S += s_part[i];
+    float T = noise[row] * S;
+    // first thread range whose running sum passes T
+    float run = 0.f;
+    int th = -1;
+    for (int i = 0; i < kSelThreads; ++i) {
+      if (run + s_part[i] > T) { th = i; break; }
+      run += s_part[i];
+    }
+    int cstar = -1;
+    float before = 0.f;
+    if (th >= 0) {
+      int a0 = min(nchunk, th * per), a1 = min(nchunk, a0 + per);
+      float acc = run;
+      for (int c = a0; c < a1; ++c) {
+        HeadRec r = rec[c];
+        float sc = r.s * expf(r.m - M);
+        // the range's own order can round differently from its partial sum:
+        // its last chunk takes the crossing then
+        if (acc + sc > T || c == a1 - 1) { cstar = c; before = acc; break; }
+        acc += sc;
+      }
+    }
+    int fallback = 0;
+    if (cstar < 0) {
+      // no crossing at all (z near 1): the last chunk with mass, last id in it
+      cstar = nchunk - 1;
+      while (cstar > 0 && !(rec[cstar].s * expf(rec[cstar].m - M) > 0.f)) --cstar;
+      fallback = 1;
+    }
+    s_chunk = cstar;
+    s_before = before;
+    s_T = T;
+    s_redi[1] = fallback;
+  }
+  __syncthreads();
+
+  // 3) recompute chunk c*'s logits (warp 0, one id per lane) and locate
+  if (warp != 0) return;
+  const int cstar = s_chunk;
+  const int v = cstar * kChunk + lane;
+  float l = -INFINITY;
+  if (v < V) {
+    const TA* hr = head_in + (size_t)row * d;
+    const TA* wr = w_head + (size_t)v * d;
+    float acc = 0.f;
+    for (int c = 0; c < d; ++c) acc += to_f(hr[c]) * to_f(wr[c]);
+    l = acc * inv_tau;
+  }
+  float e = (v < V) ? expf(l - M) : 0.f;
+  // inclusive prefix over lanes in id order
+  float pre = e;
+  for (int o = 1; o < 32; o <<= 1) {
+    float y = __shfl_up_sync(0xffffffffu, pre, o);
+    if (lane >= o) pre += y;
+  }
+  const float Tp = s_T - s_before;
+  const bool fallback = s_redi[1] != 0;
+  unsigned hit = __ballot_sync(0xffffffffu, !fallback && (v < V) && (pre > Tp));
+  unsigned pos = __ballot_sync(0xffffffffu, (v < V) && (e > 0.f));
+  if (lane == 0) {
+    int tok;
+    if (hit) tok = cstar * kChunk + (__ffs(hit) - 1);
+    else if (pos) tok = cstar * kChunk + (31 - __clz(pos));
+    else tok = min(V - 1, cstar * kChunk + 31);
+    tokens[row] = tok;
+  }
+}
+
+void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
+                        int d, const void* w_head, int V, float inv_tau, int map_kind,
+                        const float* noise, int32_t* tokens, cudaStream_t s) {
+  if (n_rows == 0) return;
+  if (bf16)
+    k_head_select<__nv_bfloat16><<<n_rows, kSelThreads, 0, s>>>(rec, nchunk,
+        (const __nv_bfloat16*)head_in, d, (const __nv_bfloat16*)w_head, V, inv_tau, map_kind,
+        noise, tokens);
+  else
+    k_head_select<float><<<n_rows, kSelThreads, 0, s>>>(rec, nchunk, (const float*)head_in, d,
+        (const float*)w_head, V, inv_tau, map_kind, noise, tokens);
+}
+
+// ---------------------------------------------------------------- commit
+// C <- [C; C_x]: the P pending tokens are now cached; the emitted tokens
+// become the next step's pending tokens (App. C.1 fixed stride).
+__global__ void k_commit(int B, int P, int nout, const int32_t* __restrict__ tokens,
+                         int32_t* pending, int pend_stride, int32_t* len) {
+  int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  for (int j = 0; j < nout; ++j) pending[b * pend_stride + j] = tokens[b * nout + j];
+  len[b] += P;
+}
+
+void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
+                   int32_t* d_len, cudaStream_t s) {
+  int nout = k > 0 ? k : 1;
+  k_commit<<<ceil_div(B, 128), 128, 0, s>>>(B, P, nout, tokens, pending, pend_stride, d_len);
+}
+
+}  // namespace kf
+
+namespace kf {
+
+// fp32 -> storage type (round to nearest even for bf16)
+template <typename T>
+__global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, size_t n) {
+  size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (; i < n; i += stride) dst[i] = from_f<T>(src[i]);
+}
+
+void launch_convert_f32(bool bf16, const float* src, void* dst, size_t n, cudaStream_t s) {
+  if (n == 0) return;
+  int blocks = (int)std::min<size_t>((n + 255) / 256, 65535);
+  if (bf16) k_convert<__nv_bfloat16><<<blocks, 256, 0, s>>>(src, (__nv_bfloat16*)dst, n);
+  else k_convert<float><<<blocks, 256, 0, s>>>(src, (float*)dst, n);
+}
+
+}  // namespace kf

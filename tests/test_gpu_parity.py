@@ -1,0 +1,271 @@
+"""GPU path vs the CPU oracle, through the C ABI (needs a GB300).
+
+fp32 model: tokens identical in every slot, logits within 1e-4.
+bf16 models: logits within 3e-2 of the oracle row's range; each differing
+token explained by the logit error (tests/parity.py).  The oracle is
+teacher-forced with the GPU's tokens after each step, so both sides always
+decode from the same context.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from synth import LM1B, OWT, TINY, make_noise, make_prompt_lengths, make_prompts, make_weights
+
+from parity import LOGIT_TOL, compare_tokens, logit_check
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def kf():
+    import __graft_entry__ as g
+    g.build()
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_10820_gb300 import kforcing
+    return kforcing
+
+
+def _run(kf, cfg, w, prompts, ks, max_k, seed=2, flags=0, map_dtype=np.float32, dec=None,
+         check_logits=True):
+    """Decode ks steps on both sides; returns per-step records."""
+    B = len(prompts)
+    if dec is None:
+        dec = kf.Decoder(cfg, w, max_batch=B, max_k=max_k, flags=flags)
+    dec.prefill(prompts)
+    ref = oracle.OracleDecoder(oracle.OracleModel(cfg, w), map_dtype=map_dtype)
+    ref.prefill(prompts)
+    rng = np.random.default_rng(seed)
+    out = []
+    for k in ks:
+        z = rng.random((B, max(k, 1)), dtype=np.float32)
+        gt = dec.step(k, z)
+        gl = dec.logits(max(k, 1)) if check_logits else None
+        rt, rl = ref.step(k, z, want_logits=True)
+        out.append((k, z, gt.copy(), rt.copy(), gl, rl))
+        # teacher-force: the oracle continues from the GPU's tokens
+        for b in range(B):
+            ref.seqs[b]["pending"] = [int(t) for t in gt[b]]
+        assert list(dec.lengths()) == [ref.cached_len(b) for b in range(B)]
+    return dec, out
+
+
+def test_tiny_fp32_tokens_identical(kf):
+    cfg = TINY
+    w = make_weights(cfg)
+    prompts = make_prompts([32, 32], cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [2, 2, 2, 1, 0, 2, 0, 0, 2], max_k=2)
+    for k, z, gt, rt, gl, rl in recs:
+        assert np.array_equal(gt, rt.astype(np.int32)), (k, gt, rt)
+        assert np.abs(gl - rl).max() < 1e-4
+    dec.close()
+
+
+def test_tiny_fp32_ragged_prompts_argmax(kf):
+    cfg = TINY.replace(map="argmax")
+    w = make_weights(cfg)
+    prompts = make_prompts([1, 7, 16, 17, 33], cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 3, 0, 4], max_k=4)
+    for k, z, gt, rt, gl, rl in recs:
+        assert np.array_equal(gt, rt.astype(np.int32)), (k, gt, rt)
+    dec.close()
+
+
+def test_tiny_fp32_rope_prefill_chunks(kf):
+    """RoPE variant with prefill split over several chunks and groups."""
+    cfg = TINY.replace(pos="rope")
+    w = make_weights(cfg)
+    prompts = make_prompts([40, 5, 23], cfg.vocab)
+    dec = kf.Decoder(cfg, w, max_batch=3, max_k=4, prefill_rows=16)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 0, 1], max_k=4, dec=dec)
+    for k, z, gt, rt, gl, rl in recs:
+        assert np.array_equal(gt, rt.astype(np.int32)), (k, gt, rt)
+        assert np.abs(gl - rl).max() < 1e-4
+    dec.close()
+
+
+def test_k_prefix_invariance_fp32(kf):
+    """A k=2 step equals the first two slots of a k=4 step (Sec. 3.4)."""
+    cfg = TINY
+    w = make_weights(cfg)
+    prompts = make_prompts([20, 20], cfg.vocab)
+    z = make_noise(1, 2, 4)[0]
+    d4 = kf.Decoder(cfg, w, max_batch=2, max_k=4)
+    d4.prefill(prompts)
+    t4 = d4.step(4, z)
+    l4 = d4.logits(4)
+    d4.rewind()
+    t2 = d4.step(2, np.ascontiguousarray(z[:, :2]))
+    l2 = d4.logits(2)
+    assert np.array_equal(t2, t4[:, :2])
+    np.testing.assert_array_equal(l2, l4[:, :2])
+    d4.close()
+
+
+def test_rewind_and_stale_noise_kv(kf):
+    """After a k=8 step wrote noise KV deep into the cache, rewinding and
+    decoding again matches a fresh context: stale noise entries are never read."""
+    cfg = TINY
+    w = make_weights(cfg)
+    prompts = make_prompts([10, 12], cfg.vocab)
+    zs = make_noise(3, 2, 8)
+    d = kf.Decoder(cfg, w, max_batch=2, max_k=8)
+    d.prefill(prompts)
+    d.step(8, zs[0])
+    d.step(8, zs[1])
+    d.rewind()
+    a = [d.step(3, np.ascontiguousarray(zs[2][:, :3])), d.step(2, np.ascontiguousarray(zs[2][:, :2]))]
+    f = kf.Decoder(cfg, w, max_batch=2, max_k=8)
+    f.prefill(prompts)
+    b = [f.step(3, np.ascontiguousarray(zs[2][:, :3])), f.step(2, np.ascontiguousarray(zs[2][:, :2]))]
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+    d.close()
+    f.close()
+
+
+def test_graph_equals_eager(kf):
+    cfg = TINY
+    w = make_weights(cfg)
+    prompts = make_prompts([9, 30], cfg.vocab)
+    zs = make_noise(4, 2, 2)
+    res = []
+    for flags in (0, kf.KF_FLAG_NO_GRAPH):
+        d = kf.Decoder(cfg, w, max_batch=2, max_k=2, flags=flags)
+        d.prefill(prompts)
+        res.append([d.step(2, zs[i]).copy() for i in range(4)])
+        d.close()
+    for a, b in zip(*res):
+        assert np.array_equal(a, b)
+
+
+def test_device_buffers(kf):
+    import torch
+    cfg = TINY
+    w = make_weights(cfg)
+    prompts = make_prompts([9, 30], cfg.vocab)
+    z = make_noise(1, 2, 2)[0]
+    d = kf.Decoder(cfg, w, max_batch=2, max_k=2)
+    d.prefill(prompts)
+    host = d.step(2, z)
+    d.rewind()
+    zd = torch.from_numpy(z).cuda()
+    od = torch.zeros((2, 2), dtype=torch.int32, device="cuda")
+    d.step(2, zd, out=od)
+    torch.cuda.synchronize()
+    d.sync()
+    assert np.array_equal(od.cpu().numpy(), host)
+    d.close()
+
+
+def test_errors_are_reported(kf):
+    cfg = TINY
+    w = make_weights(cfg)
+    d = kf.Decoder(cfg, w, max_batch=2, max_k=2)
+    z = np.zeros((2, 2), np.float32)
+    with pytest.raises(kf.KfError) as e:
+        d.B = 2
+        d.step(2, z)
+    assert e.value.code == kf.KF_E_STATE
+    d.prefill(make_prompts([60, 3], cfg.vocab))
+    with pytest.raises(kf.KfError) as e:
+        d.step(3, np.zeros((2, 3), np.float32))
+    assert e.value.code == kf.KF_E_ARG
+    d.step(2, z)          # cached 59, writes positions 59..61 of max_len 64
+    d.step(2, z)          # cached 60, writes positions 60..63
+    with pytest.raises(kf.KfError) as e:
+        d.step(2, z)      # cached 62 would write up to position 65
+    assert e.value.code == kf.KF_E_CAPACITY
+    with pytest.raises(kf.KfError) as e:
+        d.prefill(make_prompts([64], cfg.vocab))
+    assert e.value.code == kf.KF_E_CAPACITY
+    d.close()
+
+
+def _bf16_check(recs, map_kind="icdf"):
+    worst, slots, mism, bad = 0.0, 0, 0, 0
+    for k, z, gt, rt, gl, rl in recs:
+        worst = max(worst, logit_check(gl, rl))
+        n, m, u = compare_tokens(gt, rt, gl, rl, z, map_kind)
+        slots, mism, bad = slots + n, mism + m, bad + u
+    return worst, slots, mism, bad
+
+
+@pytest.fixture(scope="module")
+def lm1b_weights():
+    return make_weights(LM1B)
+
+
+def test_lm1b_bf16_small_batch(kf, lm1b_weights):
+    cfg = LM1B
+    prompts = make_prompts([32, 32, 32], cfg.vocab)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 4, 2, 0, 4], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    print(f"lm1b bf16: worst |dlogit|/range {worst:.2e}, {mism}/{slots} tokens differ, "
+          f"{bad} unexplained")
+    assert worst <= LOGIT_TOL
+    assert bad == 0
+    dec.close()
+
+
+def test_lm1b_bf16_argmax(kf, lm1b_weights):
+    cfg = LM1B.replace(map="argmax")
+    prompts = make_prompts([32, 20], cfg.vocab)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 0], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs, "argmax")
+    assert worst <= LOGIT_TOL
+    assert bad == 0
+    assert mism <= max(1, slots // 100)
+    dec.close()
+
+
+def test_lm1b_bf16_sharp_temperature(kf, lm1b_weights):
+    """At tau = 0.1 the softmax is sharp and the token agreement is >= 99.9%
+    whenever the margin exceeds the logit error (every mismatch explained)."""
+    cfg = LM1B.replace(tau=0.1)
+    prompts = make_prompts([32] * 4, cfg.vocab)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 4, 4], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    print(f"lm1b tau=0.1: {mism}/{slots} differ, {bad} unexplained")
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
+
+
+def test_lm1b_full_batch_sampled(kf, lm1b_weights):
+    """The bench's shape (batch 64, k=4, graph replay): sampled sequences
+    against the oracle, which runs only those sequences."""
+    cfg = LM1B
+    B = 64
+    prompts = make_prompts([32] * B, cfg.vocab)
+    dec = kf.Decoder(cfg, lm1b_weights, max_batch=B, max_k=4)
+    dec.prefill(prompts)
+    pick = [0, 17, 42, 63]
+    ref = oracle.OracleDecoder(oracle.OracleModel(cfg, lm1b_weights))
+    ref.prefill([prompts[i] for i in pick])
+    zs = make_noise(3, B, 4)
+    worst, slots, mism, bad = 0.0, 0, 0, 0
+    for s in range(3):
+        gt = dec.step(4, zs[s])
+        gl = dec.logits(4)[pick]
+        rt, rl = ref.step(4, zs[s][pick], want_logits=True)
+        worst = max(worst, logit_check(gl, rl))
+        n, m, u = compare_tokens(gt[pick], rt, gl, rl, zs[s][pick])
+        slots, mism, bad = slots + n, mism + m, bad + u
+        for j, b in enumerate(pick):
+            ref.seqs[j]["pending"] = [int(t) for t in gt[b]]
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
+
+
+def test_owt_ragged_paged(kf):
+    """OWT-shaped vocab with ragged prompts crossing many 16-token pages."""
+    cfg = OWT.replace(n_layer=2, max_len=256)
+    w = make_weights(cfg)
+    lens = make_prompt_lengths(4, 100, 200)
+    prompts = make_prompts(lens, cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 4, 4, 4, 1, 0], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
