@@ -1,0 +1,70 @@
+"""tcgen05 GEMM (and the SIMT GEMM) against a plain PyTorch fp32 matmul of
+the same bf16 operands, through the C ABI of include/kforcing_ops.h."""
+import ctypes
+
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [
+    (1, 128, 64),        # one row, one K block
+    (5, 256, 768),       # tiny M, split-K
+    (130, 384, 768),     # ragged M across two row tiles
+    (64, 768, 3072),     # AR-step MLP-down shape, deep split-K
+    (512, 2304, 768),    # LM1B k=4 QKV
+    (320, 3072, 768),    # first-step rows (P=1), MLP-up
+    (256, 30720, 768),   # LM-head shape (vocab padded to 256)
+    (1000, 200, 128),    # N not a multiple of the tile
+    (4096, 768, 3072),   # large M
+]
+
+
+@pytest.fixture(scope="module")
+def env():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+    from paper_2606_10820_gb300 import kforcing as kf
+    lib = kf.load_library()
+    lib.kf_op_gemm_bf16.argtypes = [ctypes.c_int32] * 4 + [ctypes.c_void_p] * 4
+    lib.kf_op_gemm_bf16.restype = ctypes.c_int
+    return torch, lib
+
+
+def _run(torch, lib, impl, A, W):
+    M, K = A.shape
+    N = W.shape[0]
+    out = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    rc = lib.kf_op_gemm_bf16(impl, M, N, K, A.data_ptr(), W.data_ptr(), out.data_ptr(), None)
+    assert rc == 0
+    torch.cuda.synchronize()
+    return out
+
+
+@pytest.mark.parametrize("M,N,K", SHAPES)
+def test_gemm_matches_fp32_matmul(env, M, N, K):
+    torch, lib = env
+    g = torch.Generator(device="cuda").manual_seed(M * 7 + N * 3 + K)
+    A = (torch.randn(M, K, device="cuda", generator=g) * 0.5).to(torch.bfloat16)
+    W = (torch.randn(N, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    ref = (A.double() @ W.double().T).float()
+    scale = ref.abs().max().item()
+    for impl in (0, 1):
+        out = _run(torch, lib, impl, A, W)
+        assert torch.isfinite(out).all()
+        err = (out - ref).abs().max().item()
+        assert err <= 1e-4 * scale + 1e-6, (impl, err, scale)
+
+
+def test_gemm_repeat_is_deterministic(env):
+    """Split-K partials are reduced in split order: identical bits each run."""
+    torch, lib = env
+    g = torch.Generator(device="cuda").manual_seed(1)
+    A = torch.randn(64, 3072, device="cuda", generator=g).to(torch.bfloat16)
+    W = (torch.randn(768, 3072, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    a = _run(torch, lib, 0, A, W)
+    b = _run(torch, lib, 0, A, W)
+    assert torch.equal(a, b)
