@@ -51,6 +51,7 @@ extern "C" {
 /* kf_config.flags */
 #define KF_FLAG_NO_GRAPH 1       /* launch kernels eagerly instead of replaying a CUDA graph */
 #define KF_FLAG_SIMT_GEMM 2      /* bf16 mode: use the SIMT GEMM, not tcgen05   */
+#define KF_FLAG_NO_PDL 4         /* launch without programmatic dependent launch */
 
 /*
  * Model and runtime configuration.  Table 4 gives the backbone (pre-norm
@@ -59,7 +60,7 @@ extern "C" {
  */
 typedef struct kf_config {
   int32_t n_layer;      /* L                                                  */
-  int32_t d_model;      /* d; d_model / n_head must be 64                     */
+  int32_t d_model;      /* d; head_dim = d_model / n_head must be 32 or 64    */
   int32_t n_head;       /* H                                                  */
   int32_t d_ff;         /* MLP width F                                        */
   int32_t vocab;        /* V                                                  */

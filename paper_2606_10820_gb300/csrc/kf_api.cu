@@ -16,6 +16,10 @@
 using namespace kf;
 
 namespace kf {
+thread_local bool g_pdl = false;
+}
+
+namespace kf {
 void launch_convert_f32(bool bf16, const float* src, void* dst, size_t n, cudaStream_t s);
 }
 
@@ -147,6 +151,13 @@ static int dalloc(kf_ctx* c, T** p, size_t bytes, bool zero = true) {
   } while (0)
 
 // ------------------------------------------------------------- launches
+// programmatic dependent launch for the kernels enqueued in this scope
+struct PdlScope {
+  bool prev;
+  explicit PdlScope(bool on) : prev(g_pdl) { g_pdl = on; }
+  ~PdlScope() { g_pdl = prev; }
+};
+
 static void prof_begin(kf_ctx* c, int kind) {
   if (!c->prof) return;
   if (c->ev_used + 2 > (int)c->ev.size()) return;
@@ -236,6 +247,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
 // captured once per (B, P, k) and replayed.
 static void enqueue_step(kf_ctx* c, int B, int P, int k) {
   cudaStream_t s = c->stream;
+  PdlScope pdl(!c->prof && !(c->cfg.flags & KF_FLAG_NO_PDL));
   const int d = c->d;
   const int S = P + k, R = B * S, nout = k > 0 ? k : 1, nh = B * nout;
   prof_begin(c, KF_KIND_ROWMAP);
@@ -538,9 +550,12 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
     KF_CUDA(cudaMemcpyAsync(c->row_pos, r_pos.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
     KF_CUDA(cudaMemcpyAsync(c->groups, grp.data(), grp.size() * sizeof(int4), cudaMemcpyHostToDevice,
                             c->stream));
-    launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
-                        c->x, c->d_err, c->stream);
-    enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
+    {
+      PdlScope pdl(!(c->cfg.flags & KF_FLAG_NO_PDL));
+      launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
+                          c->x, c->d_err, c->stream);
+      enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
+    }
     KF_CUDA(cudaGetLastError());
     // the host vectors are reused: wait until the copies have consumed them
     KF_CUDA(cudaStreamSynchronize(c->stream));

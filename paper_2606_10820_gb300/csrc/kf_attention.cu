@@ -2,38 +2,100 @@
 // sequence and one head per CTA against every cached key at or before each
 // row's position (the fully causal mask of Sec. 3.3 / Alg. 1: pending rows
 // and noise slots see the cache, earlier pending rows and earlier slots).
-// fp32 scores and online softmax; keys staged through shared memory with
-// 16-byte loads, 64 keys (4 pages) per tile.  With n_split > 1 each CTA
-// covers one key range and a combine kernel merges the partial softmaxes
-// in split order.
+//
+// Per CTA (128 threads), keys in tiles of 128 (8 pages):
+//   - K and V tiles stream into shared memory with 16-byte cp.async,
+//     double-buffered so the next tile loads while this one is computed;
+//   - scores: thread t owns key t and all R query rows (register-blocked);
+//   - online softmax per row (fp32), probabilities written transposed
+//     (P[key][row]) so the PV product broadcasts them;
+//   - PV: warp w accumulates keys 32w..32w+31 of every tile for all R rows,
+//     lanes along the head dims; the four warp partials are summed once at
+//     the end in a fixed order.
+// With n_split > 1 each CTA covers one key range and k_attn_combine merges
+// the partial softmaxes in split order.
 #include "kf_internal.cuh"
 
 namespace kf {
 
-template <typename T> struct Vec;
-template <> struct Vec<float> { static constexpr int N = 4; using V = float4; };
-template <> struct Vec<__nv_bfloat16> { static constexpr int N = 8; using V = uint4; };
+constexpr int kKeyTile = 128;
+constexpr int kAttnThreads = 128;
 
-__device__ __forceinline__ void unpack(const float4& v, float* o) {
-  o[0] = v.x; o[1] = v.y; o[2] = v.z; o[3] = v.w;
+template <typename TA> struct KvPad;
+template <> struct KvPad<float> { static constexpr int V = 4; };
+template <> struct KvPad<__nv_bfloat16> { static constexpr int V = 8; };
+
+__device__ __forceinline__ void load8(const float* p, float* o) {
+  float4 a = *reinterpret_cast<const float4*>(p);
+  float4 b = *reinterpret_cast<const float4*>(p + 4);
+  o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w; o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
 }
-__device__ __forceinline__ void unpack(const uint4& v, float* o) {
-  const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&v);
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float* o) {
+  uint4 v = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    float2 f = __bfloat1622float2(p[i]);
+    float2 f = __bfloat1622float2(h[i]);
     o[2 * i] = f.x;
     o[2 * i + 1] = f.y;
   }
 }
+// DPL consecutive values at p (DPL = 1 or 2)
+template <int DPL>
+__device__ __forceinline__ void loadd(const float* p, float* o) {
+  if (DPL == 2) { float2 f = *reinterpret_cast<const float2*>(p); o[0] = f.x; o[1] = f.y; }
+  else o[0] = p[0];
+}
+template <int DPL>
+__device__ __forceinline__ void loadd(const __nv_bfloat16* p, float* o) {
+  if (DPL == 2) {
+    float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+    o[0] = f.x; o[1] = f.y;
+  } else {
+    o[0] = __bfloat162float(p[0]);
+  }
+}
 
-constexpr int kKeyTile = 64;
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 template <typename TA, int HD>
-__global__ void __launch_bounds__(128) k_attention(AttnArgs a) {
-  constexpr int PD = HD / 8;   // output dims per thread in the PV product
-  using VT = typename Vec<TA>::V;
-  constexpr int VN = Vec<TA>::N;
+struct AttnSmem {
+  static constexpr int KP = HD + KvPad<TA>::V;      // padded K row (conflict-free 16B reads)
+  static constexpr size_t k_tile = (size_t)kKeyTile * KP * sizeof(TA);
+  static constexpr size_t v_tile = (size_t)kKeyTile * HD * sizeof(TA);
+  static size_t bytes(int R) {
+    size_t b = 0;
+    b += (size_t)R * HD * 4;              // Q
+    b += 2 * (k_tile + v_tile);           // K, V double buffer
+    b += (size_t)kKeyTile * R * 4;        // P^T
+    b += 2 * 4 * (size_t)R * 4;           // warp max / sum
+    return b;
+  }
+};
+
+template <typename TA, int HD, int R>
+__global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  using S = AttnSmem<TA, HD>;
+  constexpr int KP = S::KP;
+  constexpr int DPL = HD / 32;          // head dims per lane in the PV product
+  constexpr int CPR = HD * (int)sizeof(TA) / 16;   // 16-byte chunks per key row
+  extern __shared__ __align__(16) uint8_t sm[];
+  float* Qs = reinterpret_cast<float*>(sm);
+  TA* Kt = reinterpret_cast<TA*>(sm + (size_t)R * HD * 4);
+  TA* Vt = reinterpret_cast<TA*>(reinterpret_cast<uint8_t*>(Kt) + 2 * S::k_tile);
+  float* Ps = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(Vt) + 2 * S::v_tile);
+  float* red_m = Ps + kKeyTile * R;
+  float* red_s = red_m + 4 * R;
+
   const int g = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
   int b, row0, nr;
   if (a.groups) {
@@ -45,138 +107,173 @@ __global__ void __launch_bounds__(128) k_attention(AttnArgs a) {
   const int n_keys = a.row_pos[row0 + nr - 1] + 1;
   const int k_begin = split * a.keys_per_split;
   const int k_end = min(n_keys, k_begin + a.keys_per_split);
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
 
-  __shared__ float Qs[kMaxGroupRows][HD];
-  __shared__ float Ks[kKeyTile][HD + 1];
-  __shared__ __align__(16) float Vs[kKeyTile][HD];
-  __shared__ float Ps[kMaxGroupRows][kKeyTile];
-  __shared__ float s_m[kMaxGroupRows], s_l[kMaxGroupRows], s_corr[kMaxGroupRows];
-  __shared__ int s_pos[kMaxGroupRows];
-
-  const int t = threadIdx.x;
   const float scale = rsqrtf((float)HD);
-  for (int i = t; i < kMaxGroupRows * HD; i += 128) {
+  for (int i = t; i < R * HD; i += kAttnThreads) {
     int r = i / HD, dd = i % HD;
-    Qs[r][dd] = (r < nr) ? a.q[((size_t)(row0 + r) * a.H + h) * HD + dd] * scale : 0.f;
+    Qs[i] = (r < nr) ? a.q[((size_t)(row0 + r) * a.H + h) * HD + dd] * scale : 0.f;
   }
-  if (t < kMaxGroupRows) {
-    s_m[t] = -INFINITY;
-    s_l[t] = 0.f;
-    s_corr[t] = 1.f;
-    s_pos[t] = (t < nr) ? a.row_pos[row0 + t] : -1;
-  }
-  const int pr = t >> 3, pd = (t & 7) * PD;
-  float acc[PD];
+  int pos[R];
 #pragma unroll
-  for (int q = 0; q < PD; ++q) acc[q] = 0.f;
-  __syncthreads();
+  for (int r = 0; r < R; ++r) pos[r] = (r < nr) ? a.row_pos[row0 + r] : -1;
 
   const TA* kv = reinterpret_cast<const TA*>(a.kv);
   const size_t head_page = (size_t)kPage * HD;
   const size_t layer_base = (size_t)a.layer * a.n_pages * 2 * a.H * head_page;
   bool bad_page = false;
 
-  for (int kt = k_begin; kt < k_end; kt += kKeyTile) {
-    for (int e = t * VN; e < kKeyTile * HD; e += 128 * VN) {
-      int j = e / HD, dd = e % HD;
-      int key = kt + j;
-      float kf[VN], vf[VN];
-      int page = -1;
-      if (key < k_end) {
-        int pi = key / kPage;
-        page = pi < a.max_pages ? a.page_table[b * a.max_pages + pi] : -1;
-        if (page < 0 || page >= a.n_pages) { bad_page = true; page = -1; }
-      }
-      if (page >= 0) {
-        const TA* kp = kv + layer_base + (((size_t)page * 2) * a.H + h) * head_page +
-                       (size_t)(key % kPage) * HD + dd;
-        const TA* vp = kp + (size_t)a.H * head_page;
-        unpack(*reinterpret_cast<const VT*>(kp), kf);
-        unpack(*reinterpret_cast<const VT*>(vp), vf);
-      } else {
-#pragma unroll
-        for (int q = 0; q < VN; ++q) { kf[q] = 0.f; vf[q] = 0.f; }
-      }
-#pragma unroll
-      for (int q = 0; q < VN; ++q) { Ks[j][dd + q] = kf[q]; Vs[j][dd + q] = vf[q]; }
-    }
-    __syncthreads();
-    {  // scores for 8 rows x 1 key per thread
-      const int j = t & (kKeyTile - 1), rb = (t >> 6) * 8;
-      float sc[8];
-#pragma unroll
-      for (int r = 0; r < 8; ++r) sc[r] = 0.f;
-#pragma unroll 8
-      for (int dd = 0; dd < HD; ++dd) {
-        float kv_ = Ks[j][dd];
-#pragma unroll
-        for (int r = 0; r < 8; ++r) sc[r] += Qs[rb + r][dd] * kv_;
-      }
+  // issue the cp.async loads of the tile starting at key kt into buffer buf
+  auto load_tile = [&](int kt, int buf) {
+    TA* kd = Kt + (size_t)buf * kKeyTile * KP;
+    TA* vd = Vt + (size_t)buf * kKeyTile * HD;
+    for (int idx = t; idx < kKeyTile * CPR; idx += kAttnThreads) {
+      const int j = idx / CPR, c = idx - j * CPR;
       const int key = kt + j;
-#pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        bool ok = (rb + r < nr) && key < k_end && key <= s_pos[rb + r];
-        Ps[rb + r][j] = ok ? sc[r] : -INFINITY;
-      }
-    }
-    __syncthreads();
-    {  // online softmax, 4 rows per warp
-      const int w = t >> 5, lane = t & 31;
-#pragma unroll
-      for (int rr = 0; rr < 4; ++rr) {
-        const int r = w * 4 + rr;
-        float x0 = Ps[r][lane], x1 = Ps[r][lane + 32];
-        float mx = fmaxf(x0, x1);
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        const float m_old = s_m[r];
-        const float m_new = fmaxf(m_old, mx);
-        float p0 = 0.f, p1 = 0.f, corr = 1.f;
-        if (m_new != -INFINITY) {
-          p0 = expf(x0 - m_new);
-          p1 = expf(x1 - m_new);
-          corr = expf(m_old - m_new);
-        }
-        float sum = p0 + p1;
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-        Ps[r][lane] = p0;
-        Ps[r][lane + 32] = p1;
-        __syncwarp();
-        if (lane == 0) {
-          s_l[r] = s_l[r] * corr + sum;
-          s_m[r] = m_new;
-          s_corr[r] = corr;
+      const TA* src = kv;
+      int nbytes = 0;
+      if (key < k_end) {
+        const int pi = key / kPage;
+        const int page = pi < a.max_pages ? a.page_table[b * a.max_pages + pi] : -1;
+        if (page >= 0 && page < a.n_pages) {
+          src = kv + layer_base + (((size_t)page * 2) * a.H + h) * head_page +
+                (size_t)(key % kPage) * HD + c * (16 / sizeof(TA));
+          nbytes = 16;
+        } else {
+          bad_page = true;
         }
       }
+      cp_async16(static_cast<uint32_t>(__cvta_generic_to_shared(kd + (size_t)j * KP + c * (16 / sizeof(TA)))),
+                 src, nbytes);
+      cp_async16(static_cast<uint32_t>(__cvta_generic_to_shared(vd + (size_t)j * HD + c * (16 / sizeof(TA)))),
+                 src + (nbytes ? a.H * head_page : 0), nbytes);
+    }
+    cp_commit();
+  };
+
+  float m_run[R], l_run[R];
+  float acc[R][DPL];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    m_run[r] = -INFINITY;
+    l_run[r] = 0.f;
+#pragma unroll
+    for (int q = 0; q < DPL; ++q) acc[r][q] = 0.f;
+  }
+
+  const int n_tiles = k_end > k_begin ? ceil_div(k_end - k_begin, kKeyTile) : 0;
+  if (n_tiles > 0) load_tile(k_begin, 0);
+  __syncthreads();   // Q visible
+
+  for (int it = 0; it < n_tiles; ++it) {
+    const int kt = k_begin + it * kKeyTile;
+    const int buf = it & 1;
+    if (it + 1 < n_tiles) {
+      load_tile(kt + kKeyTile, buf ^ 1);
+      cp_wait<1>();
+    } else {
+      cp_wait<0>();
     }
     __syncthreads();
-    {  // O = O * corr + P V
-      const float c = s_corr[pr];
+    const TA* kb = Kt + (size_t)buf * kKeyTile * KP;
+    const TA* vb = Vt + (size_t)buf * kKeyTile * HD;
+
+    // scores: thread t <-> key kt + t, all R rows
+    float s[R];
 #pragma unroll
-      for (int q = 0; q < PD; ++q) acc[q] *= c;
-      for (int j = 0; j < kKeyTile; ++j) {
-        const float p = Ps[pr][j];
+    for (int r = 0; r < R; ++r) s[r] = 0.f;
+#pragma unroll 2
+    for (int d0 = 0; d0 < HD; d0 += 8) {
+      float k8[8];
+      load8(kb + (size_t)t * KP + d0, k8);
 #pragma unroll
-        for (int q4 = 0; q4 < PD; q4 += 4) {
-          const float4 v = *reinterpret_cast<const float4*>(&Vs[j][pd + q4]);
-          acc[q4] += p * v.x; acc[q4 + 1] += p * v.y; acc[q4 + 2] += p * v.z; acc[q4 + 3] += p * v.w;
-        }
+      for (int r = 0; r < R; ++r) {
+        float q8[8];
+        load8(Qs + r * HD + d0, q8);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) s[r] = fmaf(q8[i], k8[i], s[r]);
       }
     }
+    const int key = kt + t;
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+      if (!(key < k_end && key <= pos[r])) s[r] = -INFINITY;
+
+    // tile max per row
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float m = s[r];
+      for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+      if (lane == 0) red_m[warp * R + r] = m;
+    }
     __syncthreads();
+    float corr[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float tm = fmaxf(fmaxf(red_m[r], red_m[R + r]), fmaxf(red_m[2 * R + r], red_m[3 * R + r]));
+      float mn = fmaxf(m_run[r], tm);
+      float p = (mn == -INFINITY) ? 0.f : expf(s[r] - mn);
+      corr[r] = (mn == -INFINITY) ? 1.f : expf(m_run[r] - mn);
+      m_run[r] = mn;
+      s[r] = p;
+    }
+    // P^T[key][row]
+#pragma unroll
+    for (int r = 0; r < R; ++r) Ps[t * R + r] = s[r];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float sum = s[r];
+      for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      if (lane == 0) red_s[warp * R + r] = sum;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float ts = (red_s[r] + red_s[R + r]) + (red_s[2 * R + r] + red_s[3 * R + r]);
+      l_run[r] = l_run[r] * corr[r] + ts;
+#pragma unroll
+      for (int q = 0; q < DPL; ++q) acc[r][q] *= corr[r];
+    }
+    // PV over this warp's 32 keys of the tile
+#pragma unroll 4
+    for (int jj = 0; jj < 32; ++jj) {
+      const int j = warp * 32 + jj;
+      float v[DPL];
+      loadd<DPL>(vb + (size_t)j * HD + lane * DPL, v);
+      const float* pj = Ps + j * R;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        const float p = pj[r];
+#pragma unroll
+        for (int q = 0; q < DPL; ++q) acc[r][q] = fmaf(p, v[q], acc[r][q]);
+      }
+    }
+    __syncthreads();   // buffers are refilled next iteration
   }
   if (bad_page) atomicOr(a.d_err, kErrBadPage);
-  if (pr < nr) {
-    const int row = row0 + pr;
+
+  // sum the four warps' partial outputs (fixed order), then normalise
+  float* Ored = reinterpret_cast<float*>(Kt);      // [4][R][HD], K/V buffers are free
+#pragma unroll
+  for (int r = 0; r < R; ++r)
+#pragma unroll
+    for (int q = 0; q < DPL; ++q) Ored[((size_t)warp * R + r) * HD + lane * DPL + q] = acc[r][q];
+  __syncthreads();
+  for (int i = t; i < R * HD; i += kAttnThreads) {
+    const int r = i / HD, dd = i - r * HD;
+    if (r >= nr) continue;
+    float o = (Ored[i] + Ored[R * HD + i]) + (Ored[2 * R * HD + i] + Ored[3 * R * HD + i]);
+    float l = 0.f, m = -INFINITY;
+#pragma unroll
+    for (int rr = 0; rr < R; ++rr)
+      if (rr == r) { l = l_run[rr]; m = m_run[rr]; }
+    const int row = row0 + r;
     if (a.n_split == 1) {
-      const float inv = 1.f / s_l[pr];
-      TA* o = reinterpret_cast<TA*>(a.out) + (size_t)row * a.H * HD + h * HD + pd;
-#pragma unroll
-      for (int q = 0; q < PD; ++q) o[q] = from_f<TA>(acc[q] * inv);
+      TA* out = reinterpret_cast<TA*>(a.out) + (size_t)row * a.H * HD + h * HD + dd;
+      *out = from_f<TA>(o / l);
     } else {
-      float* o = a.part_o + (((size_t)split * a.R + row) * a.H + h) * HD + pd;
-#pragma unroll
-      for (int q = 0; q < PD; ++q) o[q] = acc[q];
-      if ((t & 7) == 0) a.part_ml[((size_t)split * a.R + row) * a.H + h] = make_float2(s_m[pr], s_l[pr]);
+      a.part_o[(((size_t)split * a.R + row) * a.H + h) * HD + dd] = o;
+      if (dd == 0) a.part_ml[((size_t)split * a.R + row) * a.H + h] = make_float2(m, l);
     }
   }
 }
@@ -184,6 +281,8 @@ __global__ void __launch_bounds__(128) k_attention(AttnArgs a) {
 // merge the split partial softmaxes of one (row, head), splits in order
 template <typename TA>
 __global__ void k_attn_combine(AttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x, h = blockIdx.y, dd = threadIdx.x;
   float M = -INFINITY;
   for (int s = 0; s < a.n_split; ++s) M = fmaxf(M, a.part_ml[((size_t)s * a.R + row) * a.H + h].x);
@@ -198,23 +297,46 @@ __global__ void k_attn_combine(AttnArgs a) {
   *o = from_f<TA>(O / L);
 }
 
+template <typename TA, int HD, int R>
+static void launch_r(const AttnArgs& a, int n_groups, cudaStream_t s) {
+  const size_t smem = AttnSmem<TA, HD>::bytes(R);
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(k_attention<TA, HD, R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    attr = true;
+  }
+  dim3 grid(n_groups, a.H, a.n_split);
+  kf_launch(k_attention<TA, HD, R>, dim3(grid), dim3(kAttnThreads), smem, s, a);
+}
+
+template <typename TA, int HD>
+static void launch_hd(const AttnArgs& a, int n_groups, int rows, cudaStream_t s) {
+  if (rows <= 1) launch_r<TA, HD, 1>(a, n_groups, s);
+  else if (rows <= 2) launch_r<TA, HD, 2>(a, n_groups, s);
+  else if (rows <= 4) launch_r<TA, HD, 4>(a, n_groups, s);
+  else if (rows <= 8) launch_r<TA, HD, 8>(a, n_groups, s);
+  else launch_r<TA, HD, 16>(a, n_groups, s);
+}
+
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, cudaStream_t s) {
   if (n_groups == 0) return;
-  dim3 grid(n_groups, a.H, a.n_split);
+  // rows per group: uniform in decode, at most 16 in prefill groups
+  const int rows = a.groups ? kMaxGroupRows : a.uniform_rows;
   if (a.hd == 64) {
-    if (bf16) k_attention<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
-    else k_attention<float, 64><<<grid, 128, 0, s>>>(a);
+    if (bf16) launch_hd<__nv_bfloat16, 64>(a, n_groups, rows, s);
+    else launch_hd<float, 64>(a, n_groups, rows, s);
   } else {
-    if (bf16) k_attention<__nv_bfloat16, 32><<<grid, 128, 0, s>>>(a);
-    else k_attention<float, 32><<<grid, 128, 0, s>>>(a);
+    if (bf16) launch_hd<__nv_bfloat16, 32>(a, n_groups, rows, s);
+    else launch_hd<float, 32>(a, n_groups, rows, s);
   }
 }
 
 void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s) {
   if (a.R == 0 || a.n_split <= 1) return;
   dim3 grid(a.R, a.H);
-  if (bf16) k_attn_combine<__nv_bfloat16><<<grid, a.hd, 0, s>>>(a);
-  else k_attn_combine<float><<<grid, a.hd, 0, s>>>(a);
+  if (bf16) kf_launch(k_attn_combine<__nv_bfloat16>, dim3(grid), dim3(a.hd), 0, s, a);
+  else kf_launch(k_attn_combine<float>, dim3(grid), dim3(a.hd), 0, s, a);
 }
 
 }  // namespace kf

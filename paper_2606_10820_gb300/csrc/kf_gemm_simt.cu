@@ -10,6 +10,8 @@ namespace kf {
 
 template <typename TA>
 __global__ void __launch_bounds__(128) k_gemm_simt(GemmDesc g) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float As[32][33];          // [row][k]
   __shared__ __align__(16) float Ws[32][132];  // [k][col]
   const int row0 = blockIdx.y * 32, col0 = blockIdx.x * 128;
@@ -54,8 +56,8 @@ __global__ void __launch_bounds__(128) k_gemm_simt(GemmDesc g) {
 void launch_gemm_simt(bool bf16, const GemmDesc& g, cudaStream_t s) {
   if (g.M == 0 || g.N == 0) return;
   dim3 grid(ceil_div(g.N, 128), ceil_div(g.M, 32));
-  if (bf16) k_gemm_simt<__nv_bfloat16><<<grid, 128, 0, s>>>(g);
-  else k_gemm_simt<float><<<grid, 128, 0, s>>>(g);
+  if (bf16) kf_launch(k_gemm_simt<__nv_bfloat16>, dim3(grid), dim3(128), 0, s, g);
+  else kf_launch(k_gemm_simt<float>, dim3(grid), dim3(128), 0, s, g);
 }
 
 }  // namespace kf

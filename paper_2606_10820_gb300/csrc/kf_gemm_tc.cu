@@ -154,16 +154,18 @@ __device__ __forceinline__ void epi_bar() {
 }
 
 // ------------------------------------------------------------ the kernel
-template <int BN, int STAGES>
+template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
           TcArgs g) {
   constexpr uint32_t A_BYTES = kBM * kBK * 2;
   constexpr uint32_t B_BYTES = BN * kBK * 2;
   constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static_assert(4 * 32 * 36 * 4 <= STAGE_BYTES, "epilogue transpose blocks live in stage 0");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment for the 128B swizzle pattern
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   // bars[0..S): full, bars[S..2S): empty, bars[2S]: accumulator ready
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
@@ -176,6 +178,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   const int kb0 = split * g.kb_per_split;
   const int kb1 = min(kb_total, kb0 + g.kb_per_split);
   const int nkb = kb1 - kb0;
+  pdl_trigger();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -201,7 +204,19 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
 
   if (warp == 0) {
     if (lane == 0) {
-      for (int i = 0; i < nkb; ++i) {
+      // Weights are constant during a step: the first stages' weight tiles
+      // stream in while the predecessor kernel finishes; the activation tiles
+      // it produces are loaded after pdl_wait.
+      const int pre = min(nkb, STAGES);
+      for (int i = 0; i < pre; ++i) {
+        const uint32_t full = smem_u32(&bars[i]);
+        mbar_expect_tx(full, STAGE_BYTES);
+        tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES, &map_w, full, (kb0 + i) * kBK, n0);
+      }
+      pdl_wait();
+      for (int i = 0; i < pre; ++i)
+        tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &map_a, smem_u32(&bars[i]), (kb0 + i) * kBK, m0);
+      for (int i = pre; i < nkb; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (i / STAGES) & 1;
         if (!mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, g.d_err)) break;
@@ -236,61 +251,113 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     // epilogue warps 2..5: TMEM lanes 32*(warp%4) .. +31
     const int quarter = warp & 3;
     const int et = threadIdx.x - 64;              // 0..127
+    pdl_wait();
     // one waiter, result broadcast: every epilogue thread takes the same path
     if (et == 0) s_flag[1] = mbar_wait(smem_u32(&bars[2 * STAGES]), 0, g.d_err) ? 1 : 0;
     epi_bar();
     const bool ready = s_flag[1] != 0;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const int row = m0 + quarter * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+    // Per epilogue warp a 32 x 36 fp32 block in the (now idle) pipeline
+    // stage 0: tcgen05.ld gives a thread one row's 32 columns; re-read with
+    // lane l on row (l / 8) + 4 i, columns 4 (l % 8) .. +3, every warp store
+    // covers four 128-byte row segments.
+    float* T = reinterpret_cast<float*>(smem) + quarter * (32 * 36);
+    const int rbase = m0 + quarter * 32;
+    const bool active = rbase < g.M;          // warp-uniform
+    const int gr = lane >> 3, gc = (lane & 7) * 4;
     if (ready) {
-      if (g.splits == 1) {
+      const int tile = m_tile * gridDim.x + n_tile;
+      bool last = true;
+      if (g.splits > 1) {
+        // this split's partial tile, [128 rows][BN] fp32
+        float* part = g.ws + ((size_t)tile * g.splits + split) * (kBM * BN) + (size_t)(quarter * 32) * BN;
+        if (active) {
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          float v[32];
-          tmem_ld32(lane_addr + c, v);
-          if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
-        }
-      } else {
-        const int tile = m_tile * gridDim.x + n_tile;
-        float* part = g.ws + ((size_t)tile * g.splits + split) * (kBM * BN) +
-                      (size_t)(quarter * 32 + lane) * BN;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-          float v[32];
-          tmem_ld32(lane_addr + c, v);
-          float4* p4 = reinterpret_cast<float4*>(part + c);
+          for (int c = 0; c < BN; c += 32) {
+            float v[32];
+            tmem_ld32(lane_addr + c, v);
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            __stcg(p4 + j, make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]));
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int rr = gr + 4 * i;
+              __stcg(reinterpret_cast<float4*>(part + (size_t)rr * BN + c + gc),
+                     *reinterpret_cast<const float4*>(T + rr * 36 + gc));
+            }
+            __syncwarp();
+          }
         }
         __threadfence();
         epi_bar();
         if (et == 0) {
           int old = atomicAdd(&g.counters[tile], 1);
-          *s_flag = (old == g.splits - 1);
+          s_flag[0] = (old == g.splits - 1);
         }
         epi_bar();
-        if (*s_flag) {
+        last = s_flag[0] != 0;
+        if (last) {
           __threadfence();
-          const float* base = g.ws + (size_t)tile * g.splits * (kBM * BN) +
-                              (size_t)(quarter * 32 + lane) * BN;
+          if (et == 0) g.counters[tile] = 0;   // re-arm for the next launch
+        }
+      }
+      if (last && active) {
+        const float* base = g.ws + (size_t)tile * g.splits * (kBM * BN) + (size_t)(quarter * 32) * BN;
 #pragma unroll 1
-          for (int c = 0; c < BN; c += 32) {
+        for (int c = 0; c < BN; c += 32) {
+          float4 f[8];
+          if (g.splits == 1) {
             float v[32];
+            tmem_ld32(lane_addr + c, v);
+            if (EPI == EPI_HEAD) {
+              const int row = rbase + lane;
+              if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
+              continue;
+            }
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = 0.f;
-            for (int s = 0; s < g.splits; ++s) {
-              const float4* p4 = reinterpret_cast<const float4*>(base + (size_t)s * (kBM * BN) + c);
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            __syncwarp();
 #pragma unroll
-              for (int j = 0; j < 8; ++j) {
-                float4 q = __ldcg(p4 + j);
-                v[4 * j] += q.x; v[4 * j + 1] += q.y; v[4 * j + 2] += q.z; v[4 * j + 3] += q.w;
+            for (int i = 0; i < 8; ++i) f[i] = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 36 + gc);
+            __syncwarp();
+          } else {
+            // sum the partials in split order (deterministic)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) f[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int sp = 0; sp < g.splits; ++sp) {
+              const float* ps = base + (size_t)sp * (kBM * BN) + c + gc;
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                float4 q = __ldcg(reinterpret_cast<const float4*>(ps + (size_t)(gr + 4 * i) * BN));
+                f[i].x += q.x; f[i].y += q.y; f[i].z += q.z; f[i].w += q.w;
               }
             }
-            if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
+            if (EPI == EPI_HEAD) {
+#pragma unroll
+              for (int i = 0; i < 8; ++i) *reinterpret_cast<float4*>(T + (gr + 4 * i) * 36 + gc) = f[i];
+              __syncwarp();
+              float v[32];
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                float4 t4 = *reinterpret_cast<const float4*>(T + lane * 36 + 4 * q);
+                v[4 * q] = t4.x; v[4 * q + 1] = t4.y; v[4 * q + 2] = t4.z; v[4 * q + 3] = t4.w;
+              }
+              __syncwarp();
+              const int row = rbase + lane;
+              if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
+              continue;
+            }
           }
-          if (et == 0) g.counters[tile] = 0;   // re-arm for the next launch
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int row = rbase + gr + 4 * i;
+            if (row < g.M) epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, f[i], g.N);
+          }
         }
       }
     }
@@ -336,11 +403,16 @@ bool tc_gemm_supported(const GemmDesc& g) {
   if (g.K % kBK || g.K == 0 || g.M <= 0 || g.N <= 0) return false;
   if ((g.lda * 2) % 16 || (g.ldw * 2) % 16) return false;
   if ((reinterpret_cast<uintptr_t>(g.A) & 15) || (reinterpret_cast<uintptr_t>(g.W) & 15)) return false;
+  // the vector epilogue writes groups of 4 columns
+  if (g.N % 4) return false;
+  const int k = g.epi.kind;
+  if ((k == EPI_STORE || k == EPI_STORE_F32 || k == EPI_BIAS_GELU) && g.epi.ldo % 4) return false;
+  if ((k == EPI_RESID || k == EPI_NOISE_OUT) && g.epi.ldx % 4) return false;
   return get_encode();
 }
 
-template <int BN, int STAGES>
-static int launch_bn(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
+template <int BN, int STAGES, int EPI>
+static int launch_epi(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
                      int* d_err, int num_sms, cudaStream_t s) {
   const int n_tiles = ceil_div(g.N, BN), m_tiles = ceil_div(g.M, kBM);
   const int tiles = n_tiles * m_tiles;
@@ -360,13 +432,28 @@ static int launch_bn(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters
   const size_t smem = (size_t)STAGES * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     attr_set = true;
   }
   dim3 grid(n_tiles, m_tiles, splits);
-  k_gemm_tc<BN, STAGES><<<grid, kThreads, smem, s>>>(ma, mw, a);
+  kf_launch(k_gemm_tc<BN, STAGES, EPI>, dim3(grid), dim3(kThreads), smem, s, ma, mw, a);
   return 0;
+}
+
+template <int BN, int STAGES>
+static int launch_bn(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
+                     int* d_err, int num_sms, cudaStream_t s) {
+  switch (g.epi.kind) {
+    case EPI_STORE: return launch_epi<BN, STAGES, EPI_STORE>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_HEAD: return launch_epi<BN, STAGES, EPI_HEAD>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+  }
+  return -1;
 }
 
 int launch_gemm_tc(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
@@ -377,7 +464,12 @@ int launch_gemm_tc(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, 
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
   }
-  return launch_bn<128, 6>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+  // wide tiles when they already fill the SMs; otherwise narrow tiles (and
+  // split-K) so that small-M projections still spread over every SM
+  const int tiles128 = ceil_div(g.N, 128) * ceil_div(g.M, kBM);
+  if (tiles128 >= num_sms)
+    return launch_bn<128, 6>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+  return launch_bn<64, 8>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
 }
 
 }  // namespace kf

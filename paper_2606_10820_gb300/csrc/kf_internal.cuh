@@ -119,17 +119,19 @@ __device__ __forceinline__ void epi_run32(const Epi& e, int row, int col0, const
     }
     case EPI_HEAD: {
       // col0 is a multiple of 32: one record for ids col0 .. col0+31 (< n_valid)
-      int nv = e.n_valid - col0;
+      const int nv = e.n_valid - col0;
       if (nv <= 0) break;
-      if (nv > 32) nv = 32;
       float m = -INFINITY;
       int a = col0;
-      for (int j = 0; j < nv; ++j) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
         float l = v[j] * e.inv_tau;
-        if (l > m) { m = l; a = col0 + j; }
+        if (j < nv && l > m) { m = l; a = col0 + j; }
       }
       float s = 0.f;
-      for (int j = 0; j < nv; ++j) s += expf(v[j] * e.inv_tau - m);
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nv) s += expf(v[j] * e.inv_tau - m);
       HeadRec r;
       r.m = m; r.s = s; r.a = a; r.pad = 0;
       e.rec[(size_t)row * e.nchunk + col0 / 32] = r;
@@ -145,7 +147,92 @@ __device__ __forceinline__ void epi_run32(const Epi& e, int row, int col0, const
   }
 }
 
+// Four consecutive output columns of one row (col % 4 == 0), for epilogues
+// whose lanes run along the columns of a row (coalesced vector stores).
+// EPI_HEAD is not handled here (it reduces over a run of 32 columns:
+// epi_run32).  Requires ldo, ldx and N to be multiples of 4.
+__device__ __forceinline__ void st_ta4(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+__device__ __forceinline__ void st_ta4(__nv_bfloat16* p, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
+template <typename TA, int EPI>
+__device__ __forceinline__ void epi_vec4(const Epi& e, int row, int col, float4 v, int N) {
+  if (col >= N) return;
+  if (EPI == EPI_STORE) {
+    st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
+  } else if (EPI == EPI_STORE_F32) {
+    *reinterpret_cast<float4*>(e.outf + (size_t)row * e.ldo + col) = v;
+  } else if (EPI == EPI_BIAS_GELU) {
+    if (e.bias) {
+      float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+      v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+    }
+    v = make_float4(gelu_tanh(v.x), gelu_tanh(v.y), gelu_tanh(v.z), gelu_tanh(v.w));
+    st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
+  } else if (EPI == EPI_RESID) {
+    float4* p = reinterpret_cast<float4*>(e.x + (size_t)row * e.ldx + col);
+    float4 x = *p;
+    *p = make_float4(x.x + v.x, x.y + v.y, x.z + v.z, x.w + v.w);
+  } else if (EPI == EPI_NOISE_OUT) {
+    const int xr = e.row_map[row];
+    if (e.bias) {
+      float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+      v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+    }
+    if (e.pos_emb) {
+      float4 q = *reinterpret_cast<const float4*>(e.pos_emb + (size_t)e.row_pos[xr] * N + col);
+      v.x += q.x; v.y += q.y; v.z += q.z; v.w += q.w;
+    }
+    *reinterpret_cast<float4*>(e.x + (size_t)xr * e.ldx + col) = v;
+  } else if (EPI == EPI_LOGITS) {
+    float* o = e.outf + (size_t)row * e.ldo + col;
+    const float t = e.inv_tau;
+    if (col + 3 < e.n_valid) {
+      o[0] = v.x * t; o[1] = v.y * t; o[2] = v.z * t; o[3] = v.w * t;
+    } else {
+      if (col < e.n_valid) o[0] = v.x * t;
+      if (col + 1 < e.n_valid) o[1] = v.y * t;
+      if (col + 2 < e.n_valid) o[2] = v.z * t;
+    }
+  }
+}
+
 // ---------------------------------------------------------------- launches
+// Programmatic dependent launch: every kernel of the step lets its successor
+// launch as soon as all of its own CTAs are resident (pdl_trigger), and
+// waits for its predecessor grid to complete and publish its writes
+// (pdl_wait) before its first access to any buffer another kernel of the
+// step reads or writes.  Every kernel waits unconditionally, so completion
+// stays ordered along the chain.  Launched without the attribute both are
+// no-ops.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+extern thread_local bool g_pdl;   // launch with the programmatic-serialization attribute
+
+template <typename... KArgs, typename... Args>
+inline void kf_launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                      Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = g_pdl ? 1 : 0;
+  cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 struct GemmDesc {
   int M, N, K;
   const void* A;   // [M][lda] storage TA

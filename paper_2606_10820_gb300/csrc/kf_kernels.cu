@@ -12,6 +12,8 @@ namespace kf {
 __global__ void k_rowmap(int B, int P, int k, const int32_t* __restrict__ len,
                          int32_t* row_seq, int32_t* row_pos, int32_t* noise_map,
                          int32_t* head_map) {
+  pdl_trigger();
+  pdl_wait();
   int r = blockIdx.x * blockDim.x + threadIdx.x;
   int S = P + k;
   if (r < B * S) {
@@ -30,7 +32,7 @@ __global__ void k_rowmap(int B, int P, int k, const int32_t* __restrict__ len,
 void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
                    int32_t* noise_map, int32_t* head_map, cudaStream_t s) {
   int n = B * (P + k);
-  k_rowmap<<<ceil_div(n, 128), 128, 0, s>>>(B, P, k, d_len, row_seq, row_pos, noise_map, head_map);
+  kf_launch(k_rowmap, dim3(ceil_div(n, 128)), dim3(128), 0, s, B, P, k, d_len, row_seq, row_pos, noise_map, head_map);
 }
 
 // ------------------------------------------------------------ embeddings
@@ -53,6 +55,8 @@ __global__ void k_embed_pending(int P, int k, const int32_t* __restrict__ pendin
                                 const TA* __restrict__ emb, const float* __restrict__ pos_emb,
                                 const int32_t* __restrict__ row_pos, int V, int d, float* x,
                                 int* d_err) {
+  pdl_trigger();
+  pdl_wait();
   int b = blockIdx.x / P, i = blockIdx.x - b * P;
   int r = b * (P + k) + i;
   embed_row<TA>(r, pending[b * pend_stride + i], row_pos[r], emb, pos_emb, V, d, x, d_err);
@@ -62,6 +66,8 @@ template <typename TA>
 __global__ void k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
                                const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
                                int V, int d, float* x, int* d_err) {
+  pdl_trigger();
+  pdl_wait();
   int r = blockIdx.x;
   embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, d_err);
 }
@@ -71,10 +77,10 @@ void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending
                           int V, int d, float* x, int* d_err, cudaStream_t s) {
   if (B * P == 0) return;
   if (bf16)
-    k_embed_pending<__nv_bfloat16><<<B * P, 128, 0, s>>>(P, k, pending, pend_stride,
+    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(128), 0, s, P, k, pending, pend_stride,
         (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
   else
-    k_embed_pending<float><<<B * P, 128, 0, s>>>(P, k, pending, pend_stride,
+    kf_launch(k_embed_pending<float>, dim3(B * P), dim3(128), 0, s, P, k, pending, pend_stride,
         (const float*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
 }
 
@@ -83,33 +89,41 @@ void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* t
                          int* d_err, cudaStream_t s) {
   if (R == 0) return;
   if (bf16)
-    k_embed_tokens<__nv_bfloat16><<<R, 128, 0, s>>>(row_tok, (const __nv_bfloat16*)tok_emb,
+    kf_launch(k_embed_tokens<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_tok, (const __nv_bfloat16*)tok_emb,
                                                     pos_emb, row_pos, V, d, x, d_err);
   else
-    k_embed_tokens<float><<<R, 128, 0, s>>>(row_tok, (const float*)tok_emb, pos_emb, row_pos, V,
+    kf_launch(k_embed_tokens<float>, dim3(R), dim3(128), 0, s, row_tok, (const float*)tok_emb, pos_emb, row_pos, V,
                                             d, x, d_err);
 }
 
 // ------------------------------------------------------- noise features
 // Sinusoidal encoding of z and of tau (Table 4), summed; argument
 // scale * u * freq[t], freq[t] = exp(-ln(1e4) t / (d/2)); [cos | sin].
-// Angles are formed in fp64 so the feature is the fp32 rounding of the
-// exact value.
+// The angle (up to scale radians) is formed and reduced modulo 2 pi in fp64
+// (a few DFMAs), then sincosf runs on the reduced fp32 angle: the feature is
+// accurate to fp32 rounding without fp64 transcendentals.
+__device__ __forceinline__ void sincos_reduced(double ang, float* s, float* c) {
+  const double two_pi = 6.283185307179586;
+  const double k = rint(ang * (1.0 / two_pi));
+  const float r = (float)fma(-k, two_pi, ang);
+  sincosf(r, s, c);
+}
+
 template <typename TA>
 __global__ void k_noise_feat(int n, const float* __restrict__ noise, const double* __restrict__ freq,
                              float tau, float scale, int d, TA* __restrict__ feat) {
+  pdl_trigger();
+  pdl_wait();
   int half = d / 2;
   int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= n * half) return;
   int r = idx / half, t = idx - r * half;
   double f = freq[t];
-  double az = (double)scale * (double)noise[r] * f;
-  double at = (double)scale * (double)tau * f;
-  double sz, cz, st, ct;
-  sincos(az, &sz, &cz);
-  sincos(at, &st, &ct);
-  feat[(size_t)r * d + t] = from_f<TA>((float)(cz + ct));
-  feat[(size_t)r * d + half + t] = from_f<TA>((float)(sz + st));
+  float sz, cz, st, ct;
+  sincos_reduced((double)scale * (double)noise[r] * f, &sz, &cz);
+  sincos_reduced((double)scale * (double)tau * f, &st, &ct);
+  feat[(size_t)r * d + t] = from_f<TA>(cz + ct);
+  feat[(size_t)r * d + half + t] = from_f<TA>(sz + st);
 }
 
 void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
@@ -117,10 +131,10 @@ void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq,
   if (n == 0) return;
   int tot = n * (d / 2);
   if (bf16)
-    k_noise_feat<__nv_bfloat16><<<ceil_div(tot, 256), 256, 0, s>>>(n, noise, freq, tau, scale, d,
+    kf_launch(k_noise_feat<__nv_bfloat16>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau, scale, d,
                                                                    (__nv_bfloat16*)feat);
   else
-    k_noise_feat<float><<<ceil_div(tot, 256), 256, 0, s>>>(n, noise, freq, tau, scale, d,
+    kf_launch(k_noise_feat<float>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau, scale, d,
                                                            (float*)feat);
 }
 
@@ -129,6 +143,8 @@ void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq,
 template <typename TA>
 __global__ void k_rmsnorm(const int32_t* __restrict__ row_map, const float* __restrict__ x, int d,
                           const float* __restrict__ g, float eps, TA* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   int r = blockIdx.x;
   int src = row_map ? row_map[r] : r;
   const float* xr = x + (size_t)src * d;
@@ -153,9 +169,9 @@ void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, in
                     const float* g, float eps, void* out, cudaStream_t s) {
   if (R == 0) return;
   if (bf16)
-    k_rmsnorm<__nv_bfloat16><<<R, 128, 0, s>>>(row_map, x, d, g, eps, (__nv_bfloat16*)out);
+    kf_launch(k_rmsnorm<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_map, x, d, g, eps, (__nv_bfloat16*)out);
   else
-    k_rmsnorm<float><<<R, 128, 0, s>>>(row_map, x, d, g, eps, (float*)out);
+    kf_launch(k_rmsnorm<float>, dim3(R), dim3(128), 0, s, row_map, x, d, g, eps, (float*)out);
 }
 
 // ------------------------------------------------------ RoPE + KV append
@@ -170,6 +186,8 @@ __global__ void k_rope_append(const TA* __restrict__ qkv, int d, int H,
                               const float* __restrict__ cos_t, const float* __restrict__ sin_t,
                               float* __restrict__ q, TA* __restrict__ kv, int layer, int n_pages,
                               const int32_t* __restrict__ page_table, int max_pages, int* d_err) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int HALF = HD / 2;
   int r = blockIdx.x;
   int h = threadIdx.x / HALF, i = threadIdx.x % HALF;
@@ -211,11 +229,11 @@ static void rope_append_hd(bool bf16, int R, const void* qkv, int d, int H, cons
                            int max_pages, int* d_err, cudaStream_t s) {
   int threads = H * (HD / 2);
   if (bf16)
-    k_rope_append<__nv_bfloat16, HD><<<R, threads, 0, s>>>((const __nv_bfloat16*)qkv, d, H,
+    kf_launch(k_rope_append<__nv_bfloat16, HD>, dim3(R), dim3(threads), 0, s, (const __nv_bfloat16*)qkv, d, H,
         row_seq, row_pos, cos_t, sin_t, q, (__nv_bfloat16*)kv, layer, n_pages, page_table,
         max_pages, d_err);
   else
-    k_rope_append<float, HD><<<R, threads, 0, s>>>((const float*)qkv, d, H, row_seq, row_pos,
+    kf_launch(k_rope_append<float, HD>, dim3(R), dim3(threads), 0, s, (const float*)qkv, d, H, row_seq, row_pos,
         cos_t, sin_t, q, (float*)kv, layer, n_pages, page_table, max_pages, d_err);
 }
 
@@ -242,11 +260,28 @@ void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
 // ARGMAX: the lowest id attaining M.
 constexpr int kSelThreads = 256;
 
+__device__ __forceinline__ void ld_vec(const float* p, float* o) {
+  float4 a = *reinterpret_cast<const float4*>(p);
+  o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+}
+__device__ __forceinline__ void ld_vec(const __nv_bfloat16* p, float* o) {
+  uint4 v = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float2 f = __bfloat1622float2(h[i]);
+    o[2 * i] = f.x;
+    o[2 * i + 1] = f.y;
+  }
+}
+
 template <typename TA>
 __global__ void __launch_bounds__(kSelThreads)
 k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
               const TA* __restrict__ w_head, int V, float inv_tau, int map_kind,
               const float* __restrict__ noise, int32_t* __restrict__ tokens) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x;
   const HeadRec* rec = rec_all + (size_t)row * nchunk;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -337,18 +372,35 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   }
   __syncthreads();
 
-  // 3) recompute chunk c*'s logits (warp 0, one id per lane) and locate
-  if (warp != 0) return;
+  // 3) recompute chunk c*'s 32 logits (each warp 4 ids, lanes along d with
+  //    16-byte loads), then warp 0 locates the token in id order
+  __shared__ float s_logit[kChunk];
   const int cstar = s_chunk;
-  const int v = cstar * kChunk + lane;
-  float l = -INFINITY;
-  if (v < V) {
+  {
     const TA* hr = head_in + (size_t)row * d;
-    const TA* wr = w_head + (size_t)v * d;
-    float acc = 0.f;
-    for (int c = 0; c < d; ++c) acc += to_f(hr[c]) * to_f(wr[c]);
-    l = acc * inv_tau;
+    constexpr int VEC = 16 / sizeof(TA);
+    for (int q = 0; q < kChunk / (kSelThreads / 32); ++q) {
+      const int jj = warp * (kChunk / (kSelThreads / 32)) + q;
+      const int v = cstar * kChunk + jj;
+      float acc = 0.f;
+      if (v < V) {
+        const TA* wr = w_head + (size_t)v * d;
+        for (int c0 = lane * VEC; c0 < d; c0 += 32 * VEC) {
+          float hv[VEC], wv[VEC];
+          ld_vec(hr + c0, hv);
+          ld_vec(wr + c0, wv);
+#pragma unroll
+          for (int i = 0; i < VEC; ++i) acc = fmaf(hv[i], wv[i], acc);
+        }
+      }
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      if (lane == 0) s_logit[jj] = (v < V) ? acc * inv_tau : -INFINITY;
+    }
   }
+  __syncthreads();
+  if (warp != 0) return;
+  const int v = cstar * kChunk + lane;
+  const float l = s_logit[lane];
   float e = (v < V) ? expf(l - M) : 0.f;
   // inclusive prefix over lanes in id order
   float pre = e;
@@ -374,11 +426,11 @@ void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, c
                         const float* noise, int32_t* tokens, cudaStream_t s) {
   if (n_rows == 0) return;
   if (bf16)
-    k_head_select<__nv_bfloat16><<<n_rows, kSelThreads, 0, s>>>(rec, nchunk,
+    kf_launch(k_head_select<__nv_bfloat16>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk,
         (const __nv_bfloat16*)head_in, d, (const __nv_bfloat16*)w_head, V, inv_tau, map_kind,
         noise, tokens);
   else
-    k_head_select<float><<<n_rows, kSelThreads, 0, s>>>(rec, nchunk, (const float*)head_in, d,
+    kf_launch(k_head_select<float>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk, (const float*)head_in, d,
         (const float*)w_head, V, inv_tau, map_kind, noise, tokens);
 }
 
@@ -387,6 +439,8 @@ void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, c
 // become the next step's pending tokens (App. C.1 fixed stride).
 __global__ void k_commit(int B, int P, int nout, const int32_t* __restrict__ tokens,
                          int32_t* pending, int pend_stride, int32_t* len) {
+  pdl_trigger();
+  pdl_wait();
   int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   for (int j = 0; j < nout; ++j) pending[b * pend_stride + j] = tokens[b * nout + j];
@@ -396,7 +450,7 @@ __global__ void k_commit(int B, int P, int nout, const int32_t* __restrict__ tok
 void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
                    int32_t* d_len, cudaStream_t s) {
   int nout = k > 0 ? k : 1;
-  k_commit<<<ceil_div(B, 128), 128, 0, s>>>(B, P, nout, tokens, pending, pend_stride, d_len);
+  kf_launch(k_commit, dim3(ceil_div(B, 128)), dim3(128), 0, s, B, P, nout, tokens, pending, pend_stride, d_len);
 }
 
 }  // namespace kf
@@ -406,6 +460,8 @@ namespace kf {
 // fp32 -> storage type (round to nearest even for bf16)
 template <typename T>
 __global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, size_t n) {
+  pdl_trigger();
+  pdl_wait();
   size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   size_t stride = (size_t)gridDim.x * blockDim.x;
   for (; i < n; i += stride) dst[i] = from_f<T>(src[i]);
@@ -414,8 +470,8 @@ __global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, si
 void launch_convert_f32(bool bf16, const float* src, void* dst, size_t n, cudaStream_t s) {
   if (n == 0) return;
   int blocks = (int)std::min<size_t>((n + 255) / 256, 65535);
-  if (bf16) k_convert<__nv_bfloat16><<<blocks, 256, 0, s>>>(src, (__nv_bfloat16*)dst, n);
-  else k_convert<float><<<blocks, 256, 0, s>>>(src, (float*)dst, n);
+  if (bf16) kf_launch(k_convert<__nv_bfloat16>, dim3(blocks), dim3(256), 0, s, src, (__nv_bfloat16*)dst, n);
+  else kf_launch(k_convert<float>, dim3(blocks), dim3(256), 0, s, src, (float*)dst, n);
 }
 
 }  // namespace kf

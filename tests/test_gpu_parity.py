@@ -141,6 +141,23 @@ def test_graph_equals_eager(kf):
         assert np.array_equal(a, b)
 
 
+def test_pdl_equals_plain_launches(kf):
+    """Programmatic dependent launch changes scheduling only, not results."""
+    cfg = LM1B.replace(n_layer=2)
+    w = make_weights(cfg)
+    prompts = make_prompts([17, 32, 5], cfg.vocab)
+    zs = make_noise(3, 3, 4)
+    res = []
+    for flags in (0, kf.KF_FLAG_NO_PDL, kf.KF_FLAG_NO_PDL | kf.KF_FLAG_NO_GRAPH):
+        d = kf.Decoder(cfg, w, max_batch=3, max_k=4, flags=flags)
+        d.prefill(prompts)
+        res.append([d.step(4, zs[i]).copy() for i in range(3)] + [d.logits(4)])
+        d.close()
+    for other in res[1:]:
+        for a, b in zip(res[0], other):
+            np.testing.assert_array_equal(a, b)
+
+
 def test_device_buffers(kf):
     import torch
     cfg = TINY
