@@ -20,12 +20,32 @@ extern "C" {
  * out[M][N] = A[M][K] . W[N][K]^T in fp32: the dense projections of the
  * backbone (Table 4: QKV, O, MLP) and the LM head are this contraction.
  * A, W: bf16, row-major, rows 16-byte aligned; K a multiple of 64 for
- * KF_GEMM_TCGEN05.  out: fp32 row-major [M][N].  The first call allocates a
- * split-K workspace that lives until process exit.  Errors: KF_E_ARG
- * (shapes / alignment), KF_E_CUDA.
+ * KF_GEMM_TCGEN05, N a multiple of 4.  out: fp32 row-major [M][N].  The first
+ * call allocates a 4-byte device error word that lives until process exit.
+ * Errors: KF_E_ARG (shapes / alignment), KF_E_CUDA.
  */
 int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, const void* A, const void* W,
                     float* out, void* stream);
+
+/*
+ * The LM head and its noise -> token map for `rows` normalised head rows,
+ * without writing logits to memory: l = x . w_head^T / tau with bf16
+ * operands and fp32 accumulation on the tensor cores; per 32-id chunk the
+ * maximum, sum of exp(l - max) and first argmax go to a record scratch
+ * buffer; then per row the token for noise[row]:
+ *   KF_MAP_ICDF:   the least id whose running softmax mass exceeds
+ *                  noise[row] (Eq. 1 with App. B's strict '>', Eq. icdf);
+ *   KF_MAP_ARGMAX: the lowest id of maximal logit (Alg. 1's arg max).
+ * x: bf16 [rows][d], w_head: bf16 [V][d], both row-major with 16-byte
+ * aligned rows, d a multiple of 64; noise: fp32 [rows] in [0,1);
+ * tokens: int32 [rows].  All device pointers.  The record scratch
+ * (rows x ceil(V/32) x 16 bytes) is allocated with cudaMalloc on first use
+ * and grown when a call needs more; it lives until process exit, and calls
+ * that overlap on the GPU share it.  Errors: KF_E_ARG, KF_E_OOM, KF_E_CUDA.
+ */
+int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const void* w_head,
+                      const float* noise, float tau, int32_t map_kind, int32_t* tokens,
+                      void* stream);
 
 #ifdef __cplusplus
 }

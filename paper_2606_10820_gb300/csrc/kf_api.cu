@@ -83,10 +83,6 @@ struct kf_ctx {
   float* part_o = nullptr;
   float2* part_ml = nullptr;
   size_t part_units = 0;
-  void* gemm_ws = nullptr;
-  size_t gemm_ws_bytes = 0;
-  int* gemm_counters = nullptr;
-  int n_counters = 0;
   int* d_err = nullptr;
   // graphs
   std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;
@@ -178,8 +174,7 @@ static void gemm(kf_ctx* c, int kind, int M, int N, int K, const void* A, int ld
   prof_begin(c, kind);
   bool use_tc = c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && tc_gemm_supported(g);
   if (use_tc)
-    launch_gemm_tc(g, c->gemm_ws, c->gemm_ws_bytes, c->gemm_counters, c->n_counters, c->d_err,
-                   c->stream);
+    launch_gemm_tc(g, c->d_err, c->stream);
   else
     launch_gemm_simt(c->bf16, g, c->stream);
   prof_end(c);
@@ -206,14 +201,27 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     prof_begin(c, KF_KIND_RMSNORM);
     launch_rmsnorm(c->bf16, R, nullptr, c->x, d, w.attn_norm, c->cfg.rms_eps, c->xn, s);
     prof_end(c);
-    Epi e;
-    e.kind = EPI_STORE; e.out = c->qkv; e.ldo = 3 * d;
-    gemm(c, KF_KIND_GEMM_QKV, R, 3 * d, d, c->xn, d, w.wqkv, d, e);
-    prof_begin(c, KF_KIND_ROPE_KV);
-    launch_rope_append(c->bf16, R, c->qkv, d, H, c->hd, c->row_seq, c->row_pos,
-                       c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr, c->rope_sin, c->q,
-                       c->kv, l, c->n_pages, c->d_page_table, c->max_pages, c->d_err, s);
-    prof_end(c);
+    // QKV projection; on the tensor-core path RoPE and the KV append run in
+    // its epilogue, otherwise in a separate kernel
+    Epi eq;
+    eq.kind = EPI_QKV; eq.q_out = c->q; eq.kv = c->kv; eq.layer = l; eq.n_pages = c->n_pages;
+    eq.H = H; eq.max_pages = c->max_pages; eq.dsec = d; eq.row_seq = c->row_seq;
+    eq.row_pos = c->row_pos; eq.page_table = c->d_page_table;
+    eq.cos_t = c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr; eq.sin_t = c->rope_sin;
+    eq.d_err = c->d_err;
+    const GemmDesc gq{R, 3 * d, d, c->xn, d, w.wqkv, d, eq};
+    if (c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && c->hd == 64 && tc_gemm_supported(gq)) {
+      gemm(c, KF_KIND_GEMM_QKV, R, 3 * d, d, c->xn, d, w.wqkv, d, eq);
+    } else {
+      Epi e;
+      e.kind = EPI_STORE; e.out = c->qkv; e.ldo = 3 * d;
+      gemm(c, KF_KIND_GEMM_QKV, R, 3 * d, d, c->xn, d, w.wqkv, d, e);
+      prof_begin(c, KF_KIND_ROPE_KV);
+      launch_rope_append(c->bf16, R, c->qkv, d, H, c->hd, c->row_seq, c->row_pos,
+                         c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr, c->rope_sin,
+                         c->q, c->kv, l, c->n_pages, c->d_page_table, c->max_pages, c->d_err, s);
+      prof_end(c);
+    }
     AttnArgs a{};
     a.q = c->q; a.kv = c->kv; a.layer = l; a.n_pages = c->n_pages; a.H = H; a.hd = c->hd;
     a.page_table = c->d_page_table; a.max_pages = c->max_pages;
@@ -221,7 +229,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     prof_begin(c, KF_KIND_ATTENTION);
-    launch_attention(c->bf16, a, n_groups, s);
+    launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
     if (n_split > 1) {
       prof_begin(c, KF_KIND_ATTN_COMBINE);
@@ -495,12 +503,6 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
   c->part_units = (size_t)4 * c->num_sms * kMaxGroupRows;
   if ((r = dalloc(c, &c->part_o, c->part_units * c->hd * 4)) ||
       (r = dalloc(c, &c->part_ml, c->part_units * sizeof(float2))))
-    return bail(r);
-  // split-K partial tiles of the tcgen05 GEMM and their arrival counters
-  c->gemm_ws_bytes = (size_t)64 << 20;
-  c->n_counters = 8192;
-  if ((r = dalloc(c, &c->gemm_ws, c->gemm_ws_bytes, false)) ||
-      (r = dalloc(c, &c->gemm_counters, (size_t)c->n_counters * 4)))
     return bail(r);
   e = cudaDeviceSynchronize();
   if (e != cudaSuccess) { cuda_fail(c, e, "init"); return bail(KF_E_CUDA); }

@@ -14,6 +14,9 @@
 //     the end in a fixed order.
 // With n_split > 1 each CTA covers one key range and k_attn_combine merges
 // the partial softmaxes in split order.
+#include <algorithm>
+#include <cstring>
+
 #include "kf_internal.cuh"
 
 namespace kf {
@@ -56,6 +59,28 @@ __device__ __forceinline__ void loadd(const __nv_bfloat16* p, float* o) {
   }
 }
 
+// packed fp32 FMA (two lanes per instruction; each lane rounds like fmaf)
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  unsigned long long A, B, C, D;
+  memcpy(&A, &a, 8); memcpy(&B, &b, 8); memcpy(&C, &c, 8);
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(D) : "l"(A), "l"(B), "l"(C));
+  float2 d;
+  memcpy(&d, &D, 8);
+  return d;
+}
+__device__ __forceinline__ void load8p(const float* p, float2* o) {
+  float4 a = *reinterpret_cast<const float4*>(p);
+  float4 b = *reinterpret_cast<const float4*>(p + 4);
+  o[0] = make_float2(a.x, a.y); o[1] = make_float2(a.z, a.w);
+  o[2] = make_float2(b.x, b.y); o[3] = make_float2(b.z, b.w);
+}
+__device__ __forceinline__ void load8p(const __nv_bfloat16* p, float2* o) {
+  uint4 v = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) o[i] = __bfloat1622float2(h[i]);
+}
+
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
                "r"(src_bytes)
@@ -70,17 +95,17 @@ struct AttnSmem {
   static constexpr int KP = HD + KvPad<TA>::V;      // padded K row (conflict-free 16B reads)
   static constexpr size_t k_tile = (size_t)kKeyTile * KP * sizeof(TA);
   static constexpr size_t v_tile = (size_t)kKeyTile * HD * sizeof(TA);
-  static size_t bytes(int R) {
+  static size_t bytes(int R, int nbuf) {
     size_t b = 0;
     b += (size_t)R * HD * 4;              // Q
-    b += 2 * (k_tile + v_tile);           // K, V double buffer
+    b += nbuf * (k_tile + v_tile);        // K, V (double-buffered when a CTA has > 1 tile)
     b += (size_t)kKeyTile * R * 4;        // P^T
     b += 2 * 4 * (size_t)R * 4;           // warp max / sum
     return b;
   }
 };
 
-template <typename TA, int HD, int R>
+template <typename TA, int HD, int R, int NBUF>
 __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
   pdl_trigger();
   pdl_wait();
@@ -91,8 +116,8 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
   extern __shared__ __align__(16) uint8_t sm[];
   float* Qs = reinterpret_cast<float*>(sm);
   TA* Kt = reinterpret_cast<TA*>(sm + (size_t)R * HD * 4);
-  TA* Vt = reinterpret_cast<TA*>(reinterpret_cast<uint8_t*>(Kt) + 2 * S::k_tile);
-  float* Ps = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(Vt) + 2 * S::v_tile);
+  TA* Vt = reinterpret_cast<TA*>(reinterpret_cast<uint8_t*>(Kt) + NBUF * S::k_tile);
+  float* Ps = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(Vt) + NBUF * S::v_tile);
   float* red_m = Ps + kKeyTile * R;
   float* red_s = red_m + 4 * R;
 
@@ -167,33 +192,38 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
 
   for (int it = 0; it < n_tiles; ++it) {
     const int kt = k_begin + it * kKeyTile;
-    const int buf = it & 1;
-    if (it + 1 < n_tiles) {
+    const int buf = (NBUF == 2) ? (it & 1) : 0;
+    if (NBUF == 2 && it + 1 < n_tiles) {
       load_tile(kt + kKeyTile, buf ^ 1);
       cp_wait<1>();
     } else {
+      if (NBUF == 1 && it > 0) load_tile(kt, 0);
       cp_wait<0>();
     }
     __syncthreads();
     const TA* kb = Kt + (size_t)buf * kKeyTile * KP;
     const TA* vb = Vt + (size_t)buf * kKeyTile * HD;
 
-    // scores: thread t <-> key kt + t, all R rows
-    float s[R];
+    // scores: thread t <-> key kt + t, all R rows; packed FMAs accumulate
+    // the even and odd head dims separately, summed at the end
+    float2 s2[R];
 #pragma unroll
-    for (int r = 0; r < R; ++r) s[r] = 0.f;
+    for (int r = 0; r < R; ++r) s2[r] = make_float2(0.f, 0.f);
 #pragma unroll 2
     for (int d0 = 0; d0 < HD; d0 += 8) {
-      float k8[8];
-      load8(kb + (size_t)t * KP + d0, k8);
+      float2 k2[4];
+      load8p(kb + (size_t)t * KP + d0, k2);
 #pragma unroll
       for (int r = 0; r < R; ++r) {
-        float q8[8];
-        load8(Qs + r * HD + d0, q8);
+        float2 q2[4];
+        load8p(Qs + r * HD + d0, q2);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) s[r] = fmaf(q8[i], k8[i], s[r]);
+        for (int i = 0; i < 4; ++i) s2[r] = ffma2(q2[i], k2[i], s2[r]);
       }
     }
+    float s[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) s[r] = s2[r].x + s2[r].y;
     const int key = kt + t;
 #pragma unroll
     for (int r = 0; r < R; ++r)
@@ -234,18 +264,27 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
 #pragma unroll
       for (int q = 0; q < DPL; ++q) acc[r][q] *= corr[r];
     }
-    // PV over this warp's 32 keys of the tile
+    // PV over this warp's 32 keys of the tile; packed FMAs over row pairs
 #pragma unroll 4
     for (int jj = 0; jj < 32; ++jj) {
       const int j = warp * 32 + jj;
       float v[DPL];
       loadd<DPL>(vb + (size_t)j * HD + lane * DPL, v);
       const float* pj = Ps + j * R;
+      if (R == 1) {
 #pragma unroll
-      for (int r = 0; r < R; ++r) {
-        const float p = pj[r];
+        for (int q = 0; q < DPL; ++q) acc[0][q] = fmaf(pj[0], v[q], acc[0][q]);
+      } else {
 #pragma unroll
-        for (int q = 0; q < DPL; ++q) acc[r][q] = fmaf(p, v[q], acc[r][q]);
+        for (int r = 0; r < R; r += 2) {
+          const float2 p2 = *reinterpret_cast<const float2*>(pj + r);
+#pragma unroll
+          for (int q = 0; q < DPL; ++q) {
+            float2 a2 = ffma2(p2, make_float2(v[q], v[q]), make_float2(acc[r][q], acc[r + 1][q]));
+            acc[r][q] = a2.x;
+            acc[r + 1][q] = a2.y;
+          }
+        }
       }
     }
     __syncthreads();   // buffers are refilled next iteration
@@ -297,38 +336,45 @@ __global__ void k_attn_combine(AttnArgs a) {
   *o = from_f<TA>(O / L);
 }
 
-template <typename TA, int HD, int R>
-static void launch_r(const AttnArgs& a, int n_groups, cudaStream_t s) {
-  const size_t smem = AttnSmem<TA, HD>::bytes(R);
+template <typename TA, int HD, int R, int NBUF>
+static void launch_rb(const AttnArgs& a, int n_groups, cudaStream_t s) {
+  const size_t smem = AttnSmem<TA, HD>::bytes(R, NBUF);
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(k_attention<TA, HD, R>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(k_attention<TA, HD, R, NBUF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     attr = true;
   }
   dim3 grid(n_groups, a.H, a.n_split);
-  kf_launch(k_attention<TA, HD, R>, dim3(grid), dim3(kAttnThreads), smem, s, a);
+  kf_launch(k_attention<TA, HD, R, NBUF>, grid, dim3(kAttnThreads), smem, s, a);
+}
+
+template <typename TA, int HD, int R>
+static void launch_r(const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s) {
+  // one K/V buffer when no CTA sees more than one tile of keys
+  if (std::min(a.keys_per_split, max_keys) <= kKeyTile) launch_rb<TA, HD, R, 1>(a, n_groups, s);
+  else launch_rb<TA, HD, R, 2>(a, n_groups, s);
 }
 
 template <typename TA, int HD>
-static void launch_hd(const AttnArgs& a, int n_groups, int rows, cudaStream_t s) {
-  if (rows <= 1) launch_r<TA, HD, 1>(a, n_groups, s);
-  else if (rows <= 2) launch_r<TA, HD, 2>(a, n_groups, s);
-  else if (rows <= 4) launch_r<TA, HD, 4>(a, n_groups, s);
-  else if (rows <= 8) launch_r<TA, HD, 8>(a, n_groups, s);
-  else launch_r<TA, HD, 16>(a, n_groups, s);
+static void launch_hd(const AttnArgs& a, int n_groups, int rows, int max_keys, cudaStream_t s) {
+  if (rows <= 1) launch_r<TA, HD, 1>(a, n_groups, max_keys, s);
+  else if (rows <= 2) launch_r<TA, HD, 2>(a, n_groups, max_keys, s);
+  else if (rows <= 4) launch_r<TA, HD, 4>(a, n_groups, max_keys, s);
+  else if (rows <= 8) launch_r<TA, HD, 8>(a, n_groups, max_keys, s);
+  else launch_r<TA, HD, 16>(a, n_groups, max_keys, s);
 }
 
-void launch_attention(bool bf16, const AttnArgs& a, int n_groups, cudaStream_t s) {
+void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s) {
   if (n_groups == 0) return;
   // rows per group: uniform in decode, at most 16 in prefill groups
   const int rows = a.groups ? kMaxGroupRows : a.uniform_rows;
   if (a.hd == 64) {
-    if (bf16) launch_hd<__nv_bfloat16, 64>(a, n_groups, rows, s);
-    else launch_hd<float, 64>(a, n_groups, rows, s);
+    if (bf16) launch_hd<__nv_bfloat16, 64>(a, n_groups, rows, max_keys, s);
+    else launch_hd<float, 64>(a, n_groups, rows, max_keys, s);
   } else {
-    if (bf16) launch_hd<__nv_bfloat16, 32>(a, n_groups, rows, s);
-    else launch_hd<float, 32>(a, n_groups, rows, s);
+    if (bf16) launch_hd<__nv_bfloat16, 32>(a, n_groups, rows, max_keys, s);
+    else launch_hd<float, 32>(a, n_groups, rows, max_keys, s);
   }
 }
 

@@ -11,10 +11,13 @@
 //               epilogue;
 //   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns per warp (one
 //               output row's run of 32 columns per thread) -> epi_run32.
-// When the output tiles cannot fill the SMs the K range is split over CTAs:
-// each split writes an fp32 partial tile; the last CTA to arrive on the
-// tile's counter sums the partials in split order (deterministic) and runs
-// the epilogue, then re-arms the counter.
+// When the output tiles cannot fill the SMs the K range is split over a
+// thread-block cluster of up to 8 CTAs (one per split): each keeps its fp32
+// partial tile in its own shared memory and, after a cluster barrier, CTA q
+// sums rows q, q+S, ... over distributed shared memory in split order
+// (deterministic) and runs the epilogue on them.
+// With programmatic dependent launch the producer streams the first stages'
+// weight tiles before waiting for the kernel that writes the activations.
 // Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the
 // kernel flags kErrTimeout, stops issuing work and exits after freeing TMEM.
 #include <cuda.h>
@@ -36,8 +39,6 @@ struct TcArgs {
   int M, N, K;
   int kb_per_split;   // K blocks per split
   int splits;
-  float* ws;          // [tiles][splits][128][BN] fp32 partials
-  int* counters;      // [tiles]
   int* d_err;
   Epi epi;
 };
@@ -149,6 +150,27 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// all threads of all CTAs in the cluster (warps reconverged first)
+__device__ __forceinline__ void cluster_sync() {
+  __syncwarp();
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ float4 ld_dsmem4(uint32_t local_addr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(remote)
+               : "memory");
+  return v;
+}
+
 __device__ __forceinline__ void epi_bar() {
   asm volatile("bar.sync 1, 128;" ::: "memory");
 }
@@ -161,7 +183,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   constexpr uint32_t A_BYTES = kBM * kBK * 2;
   constexpr uint32_t B_BYTES = BN * kBK * 2;
   constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static_assert(4 * 32 * 36 * 4 <= STAGE_BYTES, "epilogue transpose blocks live in stage 0");
+  static_assert(4 * 32 * 68 * 4 <= STAGES * STAGE_BYTES && kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
+                "epilogue blocks and split partials live in the idle pipeline stages");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment for the 128B swizzle pattern
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -258,109 +281,117 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     const bool ready = s_flag[1] != 0;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
-    // Per epilogue warp a 32 x 36 fp32 block in the (now idle) pipeline
-    // stage 0: tcgen05.ld gives a thread one row's 32 columns; re-read with
-    // lane l on row (l / 8) + 4 i, columns 4 (l % 8) .. +3, every warp store
-    // covers four 128-byte row segments.
-    float* T = reinterpret_cast<float*>(smem) + quarter * (32 * 36);
     const int rbase = m0 + quarter * 32;
     const bool active = rbase < g.M;          // warp-uniform
-    const int gr = lane >> 3, gc = (lane & 7) * 4;
-    if (ready) {
-      const int tile = m_tile * gridDim.x + n_tile;
-      bool last = true;
+    if (ready && active) {
       if (g.splits > 1) {
-        // this split's partial tile, [128 rows][BN] fp32
-        float* part = g.ws + ((size_t)tile * g.splits + split) * (kBM * BN) + (size_t)(quarter * 32) * BN;
-        if (active) {
-#pragma unroll 1
-          for (int c = 0; c < BN; c += 32) {
-            float v[32];
-            tmem_ld32(lane_addr + c, v);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
-                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            __syncwarp();
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int rr = gr + 4 * i;
-              __stcg(reinterpret_cast<float4*>(part + (size_t)rr * BN + c + gc),
-                     *reinterpret_cast<const float4*>(T + rr * 36 + gc));
-            }
-            __syncwarp();
-          }
-        }
-        __threadfence();
-        epi_bar();
-        if (et == 0) {
-          int old = atomicAdd(&g.counters[tile], 1);
-          s_flag[0] = (old == g.splits - 1);
-        }
-        epi_bar();
-        last = s_flag[0] != 0;
-        if (last) {
-          __threadfence();
-          if (et == 0) g.counters[tile] = 0;   // re-arm for the next launch
-        }
-      }
-      if (last && active) {
-        const float* base = g.ws + (size_t)tile * g.splits * (kBM * BN) + (size_t)(quarter * 32) * BN;
+        // this split's partial: rows of the tile in the CTA's own shared
+        // memory (pitch BN + 4), reduced across the cluster below
+        float* P = reinterpret_cast<float*>(smem) + (size_t)(quarter * 32 + lane) * (BN + 4);
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
-          float4 f[8];
-          if (g.splits == 1) {
+          float v[32];
+          tmem_ld32(lane_addr + c, v);
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            *reinterpret_cast<float4*>(P + c + 4 * q) =
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
+      } else if (EPI == EPI_HEAD) {
+        // row mode: a thread reduces its row's 32-id chunks
+        const int row = rbase + lane;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(lane_addr + c, v);
+          if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
+        }
+      } else {
+        // Per epilogue warp a 32 x 68 fp32 block in the idle pipeline stages:
+        // tcgen05.ld gives a thread one row's columns; re-read with lane l on
+        // row (l / 8) + 4 i, columns 4 (l % 8) .. +3 (and + 32): every warp
+        // store covers four 128-byte row segments.
+        float* T = reinterpret_cast<float*>(smem) + quarter * (32 * 68);
+        const int gr = lane >> 3, gc = (lane & 7) * 4;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 64) {
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
             float v[32];
-            tmem_ld32(lane_addr + c, v);
-            if (EPI == EPI_HEAD) {
-              const int row = rbase + lane;
-              if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
-              continue;
-            }
+            tmem_ld32(lane_addr + c + 32 * h2, v);
 #pragma unroll
             for (int q = 0; q < 8; ++q)
-              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
+              *reinterpret_cast<float4*>(T + lane * 68 + 32 * h2 + 4 * q) =
                   make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            __syncwarp();
-#pragma unroll
-            for (int i = 0; i < 8; ++i) f[i] = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 36 + gc);
-            __syncwarp();
-          } else {
-            // sum the partials in split order (deterministic)
-#pragma unroll
-            for (int i = 0; i < 8; ++i) f[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int sp = 0; sp < g.splits; ++sp) {
-              const float* ps = base + (size_t)sp * (kBM * BN) + c + gc;
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                float4 q = __ldcg(reinterpret_cast<const float4*>(ps + (size_t)(gr + 4 * i) * BN));
-                f[i].x += q.x; f[i].y += q.y; f[i].z += q.z; f[i].w += q.w;
-              }
-            }
-            if (EPI == EPI_HEAD) {
-#pragma unroll
-              for (int i = 0; i < 8; ++i) *reinterpret_cast<float4*>(T + (gr + 4 * i) * 36 + gc) = f[i];
-              __syncwarp();
-              float v[32];
-#pragma unroll
-              for (int q = 0; q < 8; ++q) {
-                float4 t4 = *reinterpret_cast<const float4*>(T + lane * 36 + 4 * q);
-                v[4 * q] = t4.x; v[4 * q + 1] = t4.y; v[4 * q + 2] = t4.z; v[4 * q + 3] = t4.w;
-              }
-              __syncwarp();
-              const int row = rbase + lane;
-              if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
-              continue;
-            }
           }
+          __syncwarp();
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int row = rbase + gr + 4 * i;
-            if (row < g.M) epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, f[i], g.N);
+            const float4 lo = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + gc);
+            const float4 hi = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + 32 + gc);
+            if (row < g.M) {
+              if (EPI == EPI_QKV) {
+                epi_qkv<__nv_bfloat16>(g.epi, row, n0 + c, gc, lo, hi);
+              } else {
+                epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N);
+                epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
+              }
+            }
           }
+          __syncwarp();
         }
       }
     }
+  }
+  if (g.splits > 1) {
+    // split-K across the cluster (one CTA per split): partials wait in each
+    // CTA's shared memory; CTA q then reduces rows q, q + S, ... of the tile
+    // over DSMEM, adding the splits in order (deterministic), and runs the
+    // epilogue on them.  Every thread of every CTA takes both barriers.
+    cluster_sync();
+    if (warp >= 2) {
+      // this CTA's rows q, q + S, ...: each thread takes U groups of four
+      // columns at a time and issues all their DSMEM loads before the
+      // epilogue stores, so the latencies overlap
+      constexpr int U = 4;
+      constexpr int GROUPS = BN / 4;               // float4 groups per row
+      const int S = g.splits;
+      const int q = (int)cluster_rank();
+      const int et = threadIdx.x - 64;
+      const int rows_mine = (kBM - q + S - 1) / S;
+      const int items = rows_mine * GROUPS;
+      const uint32_t pbase = smem_u32(smem);
+      for (int it0 = et; it0 < items; it0 += 128 * U) {
+        float4 acc[U];
+        int row[U], gcol[U];
+        uint32_t off[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int idx = it0 + u * 128;
+          const int rr = q + S * (idx / GROUPS);
+          gcol[u] = (idx % GROUPS) * 4;
+          row[u] = (idx < items) ? m0 + rr : g.M;   // g.M marks "no item"
+          off[u] = (uint32_t)((rr * (BN + 4) + gcol[u]) * 4);
+          acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        for (int sp = 0; sp < S; ++sp) {
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            if (row[u] < g.M) {
+              const float4 v = ld_dsmem4(pbase + off[u], (uint32_t)sp);
+              acc[u].x += v.x; acc[u].y += v.y; acc[u].z += v.z; acc[u].w += v.w;
+            }
+          }
+        }
+        if (EPI != EPI_HEAD && EPI != EPI_QKV) {   // never split (host guarantees)
+#pragma unroll
+          for (int u = 0; u < U; ++u)
+            if (row[u] < g.M) epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N);
+        }
+      }
+    }
+    cluster_sync();
   }
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
@@ -403,32 +434,29 @@ bool tc_gemm_supported(const GemmDesc& g) {
   if (g.K % kBK || g.K == 0 || g.M <= 0 || g.N <= 0) return false;
   if ((g.lda * 2) % 16 || (g.ldw * 2) % 16) return false;
   if ((reinterpret_cast<uintptr_t>(g.A) & 15) || (reinterpret_cast<uintptr_t>(g.W) & 15)) return false;
-  // the vector epilogue writes groups of 4 columns
-  if (g.N % 4) return false;
+  // the vector epilogues write groups of 4 columns (the LM-head records reduce
+  // runs of 32 columns per row and take any N)
   const int k = g.epi.kind;
+  if (k != EPI_HEAD && g.N % 4) return false;
   if ((k == EPI_STORE || k == EPI_STORE_F32 || k == EPI_BIAS_GELU) && g.epi.ldo % 4) return false;
   if ((k == EPI_RESID || k == EPI_NOISE_OUT) && g.epi.ldx % 4) return false;
+  if (k == EPI_QKV && (g.N % 64 || g.epi.dsec % 64)) return false;
   return get_encode();
 }
 
 template <int BN, int STAGES, int EPI>
-static int launch_epi(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
-                     int* d_err, int num_sms, cudaStream_t s) {
+static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s) {
   const int n_tiles = ceil_div(g.N, BN), m_tiles = ceil_div(g.M, kBM);
   const int tiles = n_tiles * m_tiles;
   const int kb_total = g.K / kBK;
+  // split K over a cluster of up to 8 CTAs when the tiles alone leave SMs
+  // idle: the largest power of two that keeps one wave and two K blocks per
+  // split (odd cluster sizes measured slower)
   int splits = 1;
-  if (tiles < num_sms) splits = std::min(std::max(1, num_sms / tiles), std::max(1, kb_total / 2));
-  while (splits > 1 && ((size_t)tiles * splits * kBM * BN * 4 > ws_bytes || tiles > n_counters))
-    --splits;
+  if (EPI != EPI_HEAD && EPI != EPI_QKV)
+    while (splits < 8 && tiles * splits * 2 <= num_sms && kb_total >= splits * 4) splits *= 2;
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
-  CUtensorMap ma, mw;
-  if (!make_map(&ma, g.A, g.M, g.K, g.lda, kBM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, BN))
-    return -1;
-  TcArgs a;
-  a.M = g.M; a.N = g.N; a.K = g.K; a.kb_per_split = kbps; a.splits = splits;
-  a.ws = reinterpret_cast<float*>(ws); a.counters = counters; a.d_err = d_err; a.epi = g.epi;
   const size_t smem = (size_t)STAGES * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256;
   static bool attr_set = false;
   if (!attr_set) {
@@ -436,40 +464,90 @@ static int launch_epi(const GemmDesc& g, void* ws, size_t ws_bytes, int* counter
                          (int)smem);
     attr_set = true;
   }
-  dim3 grid(n_tiles, m_tiles, splits);
-  kf_launch(k_gemm_tc<BN, STAGES, EPI>, dim3(grid), dim3(kThreads), smem, s, ma, mw, a);
-  return 0;
+  // a cluster of `splits` CTAs must fit on one GPC
+  static int max_cluster = 0;
+  if (!max_cluster) {
+    max_cluster = 1;
+    for (int cs = 8; cs > 1; --cs) {
+      cudaLaunchConfig_t q = {};
+      q.gridDim = dim3(1, 1, cs);
+      q.blockDim = dim3(kThreads);
+      q.dynamicSmemBytes = smem;
+      cudaLaunchAttribute ca;
+      ca.id = cudaLaunchAttributeClusterDimension;
+      ca.val.clusterDim.x = 1; ca.val.clusterDim.y = 1; ca.val.clusterDim.z = cs;
+      q.attrs = &ca;
+      q.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<BN, STAGES, EPI>, &q) == cudaSuccess && n > 0) {
+        max_cluster = cs;
+        break;
+      }
+      cudaGetLastError();
+    }
+  }
+  if (splits > max_cluster) {
+    splits = max_cluster;
+    kbps = ceil_div(kb_total, splits);
+    splits = ceil_div(kb_total, kbps);
+  }
+  CUtensorMap ma, mw;
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, kBM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, BN))
+    return -1;
+  TcArgs a;
+  a.M = g.M; a.N = g.N; a.K = g.K; a.kb_per_split = kbps; a.splits = splits;
+  a.d_err = d_err; a.epi = g.epi;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_tiles, m_tiles, splits);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  if (splits > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = 1;
+    at[na].val.clusterDim.y = 1;
+    at[na].val.clusterDim.z = splits;
+    ++na;
+  }
+  if (g_pdl) {
+    at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN, STAGES, EPI>, ma, mw, a) == cudaSuccess ? 0 : -1;
 }
 
 template <int BN, int STAGES>
-static int launch_bn(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
-                     int* d_err, int num_sms, cudaStream_t s) {
+static int launch_bn(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s) {
   switch (g.epi.kind) {
-    case EPI_STORE: return launch_epi<BN, STAGES, EPI_STORE>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_HEAD: return launch_epi<BN, STAGES, EPI_HEAD>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-    case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+    case EPI_STORE: return launch_epi<BN, STAGES, EPI_STORE>(g, d_err, num_sms, s);
+    case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU>(g, d_err, num_sms, s);
+    case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID>(g, d_err, num_sms, s);
+    case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT>(g, d_err, num_sms, s);
+    case EPI_HEAD: return launch_epi<BN, STAGES, EPI_HEAD>(g, d_err, num_sms, s);
+    case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS>(g, d_err, num_sms, s);
+    case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32>(g, d_err, num_sms, s);
+    case EPI_QKV: return launch_epi<BN, STAGES, EPI_QKV>(g, d_err, num_sms, s);
   }
   return -1;
 }
 
-int launch_gemm_tc(const GemmDesc& g, void* ws, size_t ws_bytes, int* counters, int n_counters,
-                   int* d_err, cudaStream_t s) {
+int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
   static int num_sms = 0;
   if (!num_sms) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
   }
-  // wide tiles when they already fill the SMs; otherwise narrow tiles (and
-  // split-K) so that small-M projections still spread over every SM
-  const int tiles128 = ceil_div(g.N, 128) * ceil_div(g.M, kBM);
-  if (tiles128 >= num_sms)
-    return launch_bn<128, 6>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
-  return launch_bn<64, 8>(g, ws, ws_bytes, counters, n_counters, d_err, num_sms, s);
+  // 64-wide tiles when they fit in one wave, else 128-wide (a second partial
+  // wave costs more than the wider tile)
+  const int tiles64 = ceil_div(g.N, 64) * ceil_div(g.M, kBM);
+  if (tiles64 <= num_sms) return launch_bn<64, 8>(g, d_err, num_sms, s);
+  return launch_bn<128, 6>(g, d_err, num_sms, s);
 }
 
 }  // namespace kf

@@ -51,6 +51,7 @@ enum EpiKind : int {
   EPI_HEAD = 4,       // per (row, 32-id chunk): max, sum exp(l - max), argmax of l = D/tau
   EPI_LOGITS = 5,     // outf[row][col] = D / tau     (fp32, col < n_valid)
   EPI_STORE_F32 = 6,  // outf[row][col] = D
+  EPI_QKV = 7,        // RoPE on q, k; q -> q_out (fp32), k and v -> paged KV cache
 };
 
 struct HeadRec {   // one record per (head row, chunk of 32 vocab ids)
@@ -59,6 +60,9 @@ struct HeadRec {   // one record per (head row, chunk of 32 vocab ids)
   int a;           // lowest id attaining m
   int pad;
 };
+
+__device__ __forceinline__ void st_ta4(float* p, float4 v);
+__device__ __forceinline__ void st_ta4(__nv_bfloat16* p, float4 v);
 
 struct Epi {
   int kind = EPI_STORE;
@@ -75,7 +79,57 @@ struct Epi {
   int n_valid = 0;
   HeadRec* rec = nullptr;
   int nchunk = 0;
+  // EPI_QKV
+  float* q_out = nullptr;          // [rows][H][64]
+  void* kv = nullptr;              // [L][n_pages][2][H][16][64]
+  int layer = 0, n_pages = 0, H = 0, max_pages = 0, dsec = 0;
+  const int32_t* row_seq = nullptr;
+  const int32_t* page_table = nullptr;
+  const float* cos_t = nullptr;    // [max_len][32] or NULL (no rotation)
+  const float* sin_t = nullptr;
+  int* d_err = nullptr;
 };
+
+// EPI_QKV for one row: lo = columns col0+gc .. +3 and hi = the same columns
+// + 32 of one 64-wide head block (col0 % 64 == 0, head_dim 64).  Rotates
+// the pairs (i, i + 32) of q and k at the row's position and stores q, k, v.
+template <typename TA>
+__device__ __forceinline__ void epi_qkv(const Epi& e, int row, int col0, int gc, float4 lo,
+                                        float4 hi) {
+  const int sec = col0 / e.dsec;                 // 0 q, 1 k, 2 v
+  const int h = (col0 - sec * e.dsec) >> 6;
+  const int pos = e.row_pos[row];
+  float a[4] = {lo.x, lo.y, lo.z, lo.w}, b[4] = {hi.x, hi.y, hi.z, hi.w};
+  if (sec < 2 && e.cos_t) {
+    const float4 c4 = *reinterpret_cast<const float4*>(e.cos_t + (size_t)pos * 32 + gc);
+    const float4 s4 = *reinterpret_cast<const float4*>(e.sin_t + (size_t)pos * 32 + gc);
+    const float c[4] = {c4.x, c4.y, c4.z, c4.w}, sn[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float x1 = a[j], x2 = b[j];
+      a[j] = x1 * c[j] - x2 * sn[j];
+      b[j] = x2 * c[j] + x1 * sn[j];
+    }
+  }
+  if (sec == 0) {
+    float* q = e.q_out + ((size_t)row * e.H + h) * 64 + gc;
+    *reinterpret_cast<float4*>(q) = make_float4(a[0], a[1], a[2], a[3]);
+    *reinterpret_cast<float4*>(q + 32) = make_float4(b[0], b[1], b[2], b[3]);
+    return;
+  }
+  const int bseq = e.row_seq[row];
+  const int pi = pos / kPage;
+  const int page = pi < e.max_pages ? e.page_table[bseq * e.max_pages + pi] : -1;
+  if (page < 0 || page >= e.n_pages) {
+    atomicOr(e.d_err, kErrBadPage);
+    return;
+  }
+  TA* dst = reinterpret_cast<TA*>(e.kv) +
+            ((((size_t)e.layer * e.n_pages + page) * 2 + (sec - 1)) * e.H + h) * (kPage * 64) +
+            (size_t)(pos % kPage) * 64 + gc;
+  st_ta4(dst, make_float4(a[0], a[1], a[2], a[3]));
+  st_ta4(dst + 32, make_float4(b[0], b[1], b[2], b[3]));
+}
 
 template <typename TA>
 __device__ __forceinline__ void epi_run32(const Epi& e, int row, int col0, const float* v, int N) {
@@ -247,10 +301,8 @@ void launch_gemm_simt(bool bf16, const GemmDesc& g, cudaStream_t s);
 
 // tcgen05 GEMM (bf16 only).  Requires K % 64 == 0, 16-byte aligned rows,
 // A rows readable up to round_up(M,128), W rows up to round_up(N,BN).
-struct TcPlan;
 bool tc_gemm_supported(const GemmDesc& g);
-int launch_gemm_tc(const GemmDesc& g, void* workspace, size_t ws_bytes, int* counters,
-                   int n_counters, int* d_err, cudaStream_t s);
+int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s);
 
 struct AttnArgs {
   const float* q;          // [R][H][hd] (rotated, unscaled)
@@ -270,7 +322,8 @@ struct AttnArgs {
   int keys_per_split;      // multiple of 64
   int* d_err;
 };
-void launch_attention(bool bf16, const AttnArgs& a, int n_groups, cudaStream_t s);
+// max_keys: the most keys any row of the launch can see (max_len bound)
+void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
 void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
 
 // elementwise / bookkeeping kernels

@@ -5,12 +5,40 @@
 using namespace kf;
 
 namespace {
-void* g_ws = nullptr;
-int* g_counters = nullptr;
 int* g_err = nullptr;
-constexpr size_t kWsBytes = (size_t)64 << 20;
-constexpr int kCounters = 8192;
+HeadRec* g_rec = nullptr;
+size_t g_rec_bytes = 0;
+
+int ensure_err() {
+  if (g_err) return KF_OK;
+  if (cudaMalloc(&g_err, sizeof(int)) != cudaSuccess || cudaMemset(g_err, 0, sizeof(int)) != cudaSuccess)
+    return KF_E_CUDA;
+  return KF_OK;
+}
 }  // namespace
+
+// the LM-head GEMM with the chunk-record epilogue, then the token select
+static int head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const void* w_head,
+                       const float* noise, float tau, int32_t map_kind, int32_t* tokens,
+                       HeadRec* rec, cudaStream_t s) {
+  const int nchunk = ceil_div(V, kChunk);
+  GemmDesc g{rows, V, d, x, d, w_head, d, Epi{}};
+  g.epi.kind = EPI_HEAD;
+  g.epi.inv_tau = 1.0f / tau;
+  g.epi.n_valid = V;
+  g.epi.rec = rec;
+  g.epi.nchunk = nchunk;
+  if (!tc_gemm_supported(g)) return KF_E_ARG;
+  if (launch_gemm_tc(g, g_err, s) != 0) return KF_E_CUDA;
+  launch_head_select(true, rows, rec, nchunk, x, d, w_head, V, 1.0f / tau, map_kind, noise, tokens, s);
+  return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
+}
+
+static bool head_args_ok(int32_t rows, int32_t V, int32_t d, const void* x, const void* w,
+                         const float* noise, float tau, int32_t map_kind, const int32_t* tokens) {
+  return rows > 0 && V > 0 && d > 0 && d % 64 == 0 && x && w && noise && tokens && tau > 0.f &&
+         (map_kind == KF_MAP_ICDF || map_kind == KF_MAP_ARGMAX);
+}
 
 extern "C" int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, const void* A,
                                const void* W, float* out, void* stream) {
@@ -22,19 +50,36 @@ extern "C" int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, co
   cudaStream_t s = (cudaStream_t)stream;
   if (impl == KF_GEMM_TCGEN05) {
     if (!tc_gemm_supported(g)) return KF_E_ARG;
-    if (!g_ws) {
-      if (cudaMalloc(&g_ws, kWsBytes) != cudaSuccess ||
-          cudaMalloc(&g_counters, kCounters * sizeof(int)) != cudaSuccess ||
-          cudaMalloc(&g_err, sizeof(int)) != cudaSuccess ||
-          cudaMemset(g_counters, 0, kCounters * sizeof(int)) != cudaSuccess ||
-          cudaMemset(g_err, 0, sizeof(int)) != cudaSuccess)
-        return KF_E_CUDA;
-    }
-    if (launch_gemm_tc(g, g_ws, kWsBytes, g_counters, kCounters, g_err, s) != 0) return KF_E_CUDA;
+    if (ensure_err() != KF_OK) return KF_E_CUDA;
+    if (launch_gemm_tc(g, g_err, s) != 0) return KF_E_CUDA;
   } else if (impl == KF_GEMM_SIMT) {
     launch_gemm_simt(true, g, s);
   } else {
     return KF_E_ARG;
   }
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
+}
+
+extern "C" int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void* x,
+                                 const void* w_head, const float* noise, float tau,
+                                 int32_t map_kind, int32_t* tokens, void* stream) {
+  if (!head_args_ok(rows, V, d, x, w_head, noise, tau, map_kind, tokens)) return KF_E_ARG;
+  if (ensure_err() != KF_OK) return KF_E_CUDA;
+  const size_t need = (size_t)rows * ceil_div(V, kChunk) * sizeof(HeadRec);
+  if (need > g_rec_bytes) {
+    cudaStream_t s = (cudaStream_t)stream;
+    if (g_rec) {
+      cudaStreamSynchronize(s);   // a pending call may still read the old buffer
+      cudaFree(g_rec);
+      g_rec = nullptr;
+      g_rec_bytes = 0;
+    }
+    if (cudaMalloc(&g_rec, need) != cudaSuccess) {
+      cudaGetLastError();
+      return KF_E_OOM;
+    }
+    g_rec_bytes = need;
+  }
+  return head_tokens(rows, V, d, x, w_head, noise, tau, map_kind, tokens, g_rec,
+                     (cudaStream_t)stream);
 }
