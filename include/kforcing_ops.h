@@ -47,6 +47,30 @@ int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const v
                       const float* noise, float tau, int32_t map_kind, int32_t* tokens,
                       void* stream);
 
+/*
+ * kf_op_head_tokens_noalloc: the same computation as kf_op_head_tokens, for
+ * callers that must not allocate device memory, for instance code whose
+ * device memory is fully owned by another allocator or budgeted up front,
+ * or a loop that cannot afford the device-wide synchronisation cudaMalloc and
+ * cudaFree may cause.  It calls no cudaMalloc, cudaFree or other allocating
+ * routine.  The paper has no counterpart: this is a deployment variant.
+ *
+ * Scratch: the chunk records live in a fixed array inside the library's
+ * device image, KF_NOALLOC_MAX_RECORDS records of 16 bytes (4 MiB) plus an
+ * error word; every GPU that loads the library holds it until the process
+ * exits.  A call needs rows * ceil(V/32) records; larger calls are rejected
+ * with KF_E_CAPACITY (kf_last_error(NULL) says why) before anything runs.
+ * The first call on each device, made with that device current, looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture.  All calls share the one array: calls whose work
+ * overlaps on the GPU (different streams, or other threads) race on it.
+ * Arguments, layouts and the other errors are those of kf_op_head_tokens.
+ */
+#define KF_NOALLOC_MAX_RECORDS 262144
+int kf_op_head_tokens_noalloc(int32_t rows, int32_t V, int32_t d, const void* x,
+                              const void* w_head, const float* noise, float tau,
+                              int32_t map_kind, int32_t* tokens, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

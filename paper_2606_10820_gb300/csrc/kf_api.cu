@@ -96,6 +96,10 @@ struct kf_ctx {
 
 static thread_local std::string g_err;
 
+namespace kf {
+void set_global_error(const std::string& msg) { g_err = msg; }
+}
+
 static int fail(kf_ctx* c, int code, const std::string& msg) {
   if (c) c->err = msg;
   else g_err = msg;

@@ -326,6 +326,9 @@ struct AttnArgs {
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
 void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
 
+// message for kf_last_error(NULL) (calls without a context)
+void set_global_error(const std::string& msg);
+
 // elementwise / bookkeeping kernels
 void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
                    int32_t* noise_map, int32_t* head_map, cudaStream_t s);
