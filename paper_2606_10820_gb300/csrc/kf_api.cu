@@ -69,6 +69,8 @@ struct kf_ctx {
   int pend_stride = 8;
   // workspaces
   int R_cap = 0, NR_cap = 0, prefill_rows = 0;
+  bool fused = false;     // RMSNorm fused into the tcgen05 GEMMs (bf16, head_dim 64)
+  float* ss = nullptr;    // [rows][d/64] sums of squares of the residual stream
   float* x = nullptr;
   void *xn = nullptr, *qkv = nullptr, *attn = nullptr, *hmid = nullptr;
   float* q = nullptr;
@@ -194,27 +196,38 @@ static void attn_plan(kf_ctx* c, int n_groups, int R, int* n_split, int* kps) {
   *kps = round_up(ceil_div(c->cfg.max_len, s), 64);
 }
 
-// L decoder layers over R rows (Table 4): pre-norm attention and MLP blocks
+// L decoder layers over R rows (Table 4): pre-norm attention and MLP blocks.
+// On the fused tensor-core path (c->fused) the pre-norms run inside the
+// GEMMs: xn holds bf16(x), ss the per-64-column sums of squares written by
+// the producers of x, and the QKV and MLP-up epilogues scale their rows (the
+// gains are folded into wqkv and w_up).  Otherwise an RMSNorm kernel writes
+// the normed rows into xn.
 static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, int uniform_rows) {
   const int d = c->d, H = c->H, F = c->F;
   cudaStream_t s = c->stream;
   int n_split, kps;
   attn_plan(c, n_groups, R, &n_split, &kps);
+  auto norm_in = [&](Epi& e) {
+    e.ss_in = c->ss; e.nslot = d / 64; e.inv_d = 1.0f / d; e.eps = c->cfg.rms_eps;
+  };
+  auto norm_out = [&](Epi& e) { e.xb_out = c->xn; e.ss_out = c->ss; e.nslot = d / 64; };
   for (int l = 0; l < c->L; ++l) {
     const LayerW& w = c->layers[l];
-    prof_begin(c, KF_KIND_RMSNORM);
-    launch_rmsnorm(c->bf16, R, nullptr, c->x, d, w.attn_norm, c->cfg.rms_eps, c->xn, s);
-    prof_end(c);
+    if (!c->fused) {
+      prof_begin(c, KF_KIND_RMSNORM);
+      launch_rmsnorm(c->bf16, R, nullptr, c->x, d, w.attn_norm, c->cfg.rms_eps, c->xn, s);
+      prof_end(c);
+    }
     // QKV projection; on the tensor-core path RoPE and the KV append run in
     // its epilogue, otherwise in a separate kernel
-    Epi eq;
-    eq.kind = EPI_QKV; eq.q_out = c->q; eq.kv = c->kv; eq.layer = l; eq.n_pages = c->n_pages;
-    eq.H = H; eq.max_pages = c->max_pages; eq.dsec = d; eq.row_seq = c->row_seq;
-    eq.row_pos = c->row_pos; eq.page_table = c->d_page_table;
-    eq.cos_t = c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr; eq.sin_t = c->rope_sin;
-    eq.d_err = c->d_err;
-    const GemmDesc gq{R, 3 * d, d, c->xn, d, w.wqkv, d, eq};
-    if (c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && c->hd == 64 && tc_gemm_supported(gq)) {
+    if (c->fused) {
+      Epi eq;
+      eq.kind = EPI_QKV; eq.q_out = c->q; eq.kv = c->kv; eq.layer = l; eq.n_pages = c->n_pages;
+      eq.H = H; eq.max_pages = c->max_pages; eq.dsec = d; eq.row_seq = c->row_seq;
+      eq.row_pos = c->row_pos; eq.page_table = c->d_page_table;
+      eq.cos_t = c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr; eq.sin_t = c->rope_sin;
+      eq.d_err = c->d_err;
+      norm_in(eq);
       gemm(c, KF_KIND_GEMM_QKV, R, 3 * d, d, c->xn, d, w.wqkv, d, eq);
     } else {
       Epi e;
@@ -242,15 +255,20 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     }
     Epi eo;
     eo.kind = EPI_RESID; eo.x = c->x; eo.ldx = d;
+    if (c->fused) norm_out(eo);
     gemm(c, KF_KIND_GEMM_O, R, d, d, c->attn, d, w.wo, d, eo);
-    prof_begin(c, KF_KIND_RMSNORM);
-    launch_rmsnorm(c->bf16, R, nullptr, c->x, d, w.mlp_norm, c->cfg.rms_eps, c->xn, s);
-    prof_end(c);
+    if (!c->fused) {
+      prof_begin(c, KF_KIND_RMSNORM);
+      launch_rmsnorm(c->bf16, R, nullptr, c->x, d, w.mlp_norm, c->cfg.rms_eps, c->xn, s);
+      prof_end(c);
+    }
     Epi eu;
     eu.kind = EPI_BIAS_GELU; eu.out = c->hmid; eu.ldo = F;
+    if (c->fused) norm_in(eu);
     gemm(c, KF_KIND_GEMM_UP, R, F, d, c->xn, d, w.w_up, d, eu);
     Epi ed;
     ed.kind = EPI_RESID; ed.x = c->x; ed.ldx = d;
+    if (c->fused) norm_out(ed);
     gemm(c, KF_KIND_GEMM_DOWN, R, d, F, c->hmid, F, w.w_down, F, ed);
   }
 }
@@ -267,7 +285,8 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k) {
   prof_end(c);
   prof_begin(c, KF_KIND_EMBED);
   launch_embed_pending(c->bf16, B, P, k, c->d_pending, c->pend_stride, c->tok_emb, c->pos_emb,
-                       c->row_pos, c->V, d, c->x, c->d_err, s);
+                       c->row_pos, c->V, d, c->x, c->fused ? c->xn : nullptr,
+                       c->fused ? c->ss : nullptr, c->d_err, s);
   if (k > 0)
     launch_noise_feat(c->bf16, B * k, c->noise, c->noise_freq, c->cfg.tau, c->cfg.noise_scale, d,
                       c->nfeat, s);
@@ -280,6 +299,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k) {
     Epi e2;
     e2.kind = EPI_NOISE_OUT; e2.x = c->x; e2.ldx = d; e2.bias = c->ne_b2;
     e2.row_map = c->noise_map; e2.row_pos = c->row_pos; e2.pos_emb = c->pos_emb;
+    if (c->fused) { e2.xb_out = c->xn; e2.ss_out = c->ss; e2.nslot = d / 64; }
     gemm(c, KF_KIND_NOISE_GEMM, B * k, d, c->NH, c->nhid, c->NH, c->ne_w2, c->NH, e2);
   }
   enqueue_layers(c, R, B, nullptr, S);
@@ -401,10 +421,13 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
                                (size_t)NH * d, (size_t)cfg.max_len * d});
   float* stage = nullptr;
   if ((r = dalloc(c, &stage, max_elems * 4, false))) return bail(r);
+  const float* fold_gain = nullptr;   // gains to fold into the columns being uploaded
+  int fold_rows = 0;
   auto upload = [&](const float* src, size_t n, void* dst, bool convert) -> int {
     e = cudaMemcpyAsync(stage, src, n * 4, dev_w ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice,
                         c->stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "weight copy");
+    if (fold_gain) launch_scale_cols(stage, fold_gain, fold_rows, d, n, c->stream);
     if (convert) launch_convert_f32(c->bf16, stage, dst, n, c->stream);
     else launch_convert_f32(false, stage, dst, n, c->stream);
     e = cudaStreamSynchronize(c->stream);
@@ -422,12 +445,25 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
         (r = upload(w->pos_emb, (size_t)cfg.max_len * d, c->pos_emb, false)))
       return bail(r);
   }
-  if ((r = wbuf(&wqkv, (size_t)L * 3 * d * d)) || (r = upload(w->wqkv, (size_t)L * 3 * d * d, wqkv, true)) ||
-      (r = wbuf(&wo, (size_t)L * d * d)) || (r = upload(w->wo, (size_t)L * d * d, wo, true)) ||
-      (r = wbuf(&wup, (size_t)L * F * d)) || (r = upload(w->w_up, (size_t)L * F * d, wup, true)) ||
-      (r = wbuf(&wdown, (size_t)L * d * F)) || (r = upload(w->w_down, (size_t)L * d * F, wdown, true)) ||
-      (r = fbuf(&an, (size_t)L * d)) || (r = upload(w->attn_norm, (size_t)L * d, an, false)) ||
+  // the fused path folds the pre-norm gains into the consuming projections:
+  // rmsnorm(x) W^T = rinv(x) * (x (W diag(g))^T)
+  c->fused = c->bf16 && !(cfg.flags & KF_FLAG_SIMT_GEMM) && c->hd == 64 && d % 64 == 0;
+  auto upload_fold = [&](const float* src, size_t n, void* dst, const float* gains,
+                         int rows_per_layer) -> int {
+    fold_gain = gains;
+    fold_rows = rows_per_layer;
+    int rr = upload(src, n, dst, true);
+    fold_gain = nullptr;
+    return rr;
+  };
+  if ((r = fbuf(&an, (size_t)L * d)) || (r = upload(w->attn_norm, (size_t)L * d, an, false)) ||
       (r = fbuf(&mn, (size_t)L * d)) || (r = upload(w->mlp_norm, (size_t)L * d, mn, false)) ||
+      (r = wbuf(&wqkv, (size_t)L * 3 * d * d)) ||
+      (r = upload_fold(w->wqkv, (size_t)L * 3 * d * d, wqkv, c->fused ? an : nullptr, 3 * d)) ||
+      (r = wbuf(&wo, (size_t)L * d * d)) || (r = upload(w->wo, (size_t)L * d * d, wo, true)) ||
+      (r = wbuf(&wup, (size_t)L * F * d)) ||
+      (r = upload_fold(w->w_up, (size_t)L * F * d, wup, c->fused ? mn : nullptr, F)) ||
+      (r = wbuf(&wdown, (size_t)L * d * F)) || (r = upload(w->w_down, (size_t)L * d * F, wdown, true)) ||
       (r = fbuf(&c->final_norm, d)) || (r = upload(w->final_norm, d, c->final_norm, false)) ||
       (r = wbuf(&c->w_head, (size_t)c->V_pad * d)) ||
       (r = upload(w->w_head, (size_t)V * d, c->w_head, true)) ||
@@ -491,6 +527,7 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
       (r = dalloc(c, &c->d_pending, (size_t)MB * MK * 4)) ||
       (r = dalloc(c, &c->d_pending0, (size_t)MB * MK * 4)) ||
       (r = dalloc(c, &c->x, (size_t)R * d * 4)) || (r = wbuf(&c->xn, (size_t)R * d)) ||
+      (r = dalloc(c, &c->ss, (size_t)R * (d / 64 + 1) * 4)) ||
       (r = wbuf(&c->qkv, (size_t)R * 3 * d)) || (r = dalloc(c, &c->q, (size_t)R * d * 4)) ||
       (r = wbuf(&c->attn, (size_t)R * d)) || (r = wbuf(&c->hmid, (size_t)R * F)) ||
       (r = wbuf(&c->nfeat, (size_t)c->NR_cap * d)) || (r = wbuf(&c->nhid, (size_t)c->NR_cap * NH)) ||
@@ -559,7 +596,8 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
     {
       PdlScope pdl(!(c->cfg.flags & KF_FLAG_NO_PDL));
       launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
-                          c->x, c->d_err, c->stream);
+                          c->x, c->fused ? c->xn : nullptr, c->fused ? c->ss : nullptr, c->d_err,
+                          c->stream);
       enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
     }
     KF_CUDA(cudaGetLastError());

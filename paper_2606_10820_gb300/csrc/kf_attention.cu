@@ -134,11 +134,6 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
   const int k_end = min(n_keys, k_begin + a.keys_per_split);
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
 
-  const float scale = rsqrtf((float)HD);
-  for (int i = t; i < R * HD; i += kAttnThreads) {
-    int r = i / HD, dd = i % HD;
-    Qs[i] = (r < nr) ? a.q[((size_t)(row0 + r) * a.H + h) * HD + dd] * scale : 0.f;
-  }
   int pos[R];
 #pragma unroll
   for (int r = 0; r < R; ++r) pos[r] = (r < nr) ? a.row_pos[row0 + r] : -1;
@@ -176,18 +171,30 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
     cp_commit();
   };
 
+  // running max / sum per row; the PV accumulators hold row pairs (r, r+1)
+  // of head dims lane*DPL + q, so a packed FMA updates both rows at once
+  constexpr int RP = (R + 1) / 2;
   float m_run[R], l_run[R];
-  float acc[R][DPL];
+  float2 acc2[RP][DPL];
 #pragma unroll
   for (int r = 0; r < R; ++r) {
     m_run[r] = -INFINITY;
     l_run[r] = 0.f;
-#pragma unroll
-    for (int q = 0; q < DPL; ++q) acc[r][q] = 0.f;
   }
+#pragma unroll
+  for (int rp = 0; rp < RP; ++rp)
+#pragma unroll
+    for (int q = 0; q < DPL; ++q) acc2[rp][q] = make_float2(0.f, 0.f);
 
   const int n_tiles = k_end > k_begin ? ceil_div(k_end - k_begin, kKeyTile) : 0;
-  if (n_tiles > 0) load_tile(k_begin, 0);
+  if (n_tiles > 0) load_tile(k_begin, 0);   // first K/V tile in flight while Q loads
+  const float scale = rsqrtf((float)HD);
+  for (int i = t * 4; i < R * HD; i += kAttnThreads * 4) {
+    const int r = i / HD, dd = i % HD;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (r < nr) v = *reinterpret_cast<const float4*>(a.q + ((size_t)(row0 + r) * a.H + h) * HD + dd);
+    *reinterpret_cast<float4*>(Qs + i) = make_float4(v.x * scale, v.y * scale, v.z * scale, v.w * scale);
+  }
   __syncthreads();   // Q visible
 
   for (int it = 0; it < n_tiles; ++it) {
@@ -248,8 +255,14 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
       s[r] = p;
     }
     // P^T[key][row]
+    if (R % 4 == 0) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) Ps[t * R + r] = s[r];
+      for (int r = 0; r < R; r += 4)
+        *reinterpret_cast<float4*>(Ps + t * R + r) = make_float4(s[r], s[r + 1], s[r + 2], s[r + 3]);
+    } else {
+#pragma unroll
+      for (int r = 0; r < R; ++r) Ps[t * R + r] = s[r];
+    }
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       float sum = s[r];
@@ -261,8 +274,15 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
     for (int r = 0; r < R; ++r) {
       float ts = (red_s[r] + red_s[R + r]) + (red_s[2 * R + r] + red_s[3 * R + r]);
       l_run[r] = l_run[r] * corr[r] + ts;
+    }
 #pragma unroll
-      for (int q = 0; q < DPL; ++q) acc[r][q] *= corr[r];
+    for (int rp = 0; rp < RP; ++rp) {
+      const float c0 = corr[2 * rp], c1 = (2 * rp + 1 < R) ? corr[2 * rp + 1] : 1.f;
+#pragma unroll
+      for (int q = 0; q < DPL; ++q) {
+        acc2[rp][q].x *= c0;
+        acc2[rp][q].y *= c1;
+      }
     }
     // PV over this warp's 32 keys of the tile; packed FMAs over row pairs
 #pragma unroll 4
@@ -273,17 +293,13 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
       const float* pj = Ps + j * R;
       if (R == 1) {
 #pragma unroll
-        for (int q = 0; q < DPL; ++q) acc[0][q] = fmaf(pj[0], v[q], acc[0][q]);
+        for (int q = 0; q < DPL; ++q) acc2[0][q].x = fmaf(pj[0], v[q], acc2[0][q].x);
       } else {
 #pragma unroll
-        for (int r = 0; r < R; r += 2) {
-          const float2 p2 = *reinterpret_cast<const float2*>(pj + r);
+        for (int rp = 0; rp < RP; ++rp) {
+          const float2 p2 = *reinterpret_cast<const float2*>(pj + 2 * rp);
 #pragma unroll
-          for (int q = 0; q < DPL; ++q) {
-            float2 a2 = ffma2(p2, make_float2(v[q], v[q]), make_float2(acc[r][q], acc[r + 1][q]));
-            acc[r][q] = a2.x;
-            acc[r + 1][q] = a2.y;
-          }
+          for (int q = 0; q < DPL; ++q) acc2[rp][q] = ffma2(p2, make_float2(v[q], v[q]), acc2[rp][q]);
         }
       }
     }
@@ -294,9 +310,12 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
   // sum the four warps' partial outputs (fixed order), then normalise
   float* Ored = reinterpret_cast<float*>(Kt);      // [4][R][HD], K/V buffers are free
 #pragma unroll
-  for (int r = 0; r < R; ++r)
+  for (int rp = 0; rp < RP; ++rp)
 #pragma unroll
-    for (int q = 0; q < DPL; ++q) Ored[((size_t)warp * R + r) * HD + lane * DPL + q] = acc[r][q];
+    for (int q = 0; q < DPL; ++q) {
+      Ored[((size_t)warp * R + 2 * rp) * HD + lane * DPL + q] = acc2[rp][q].x;
+      if (2 * rp + 1 < R) Ored[((size_t)warp * R + 2 * rp + 1) * HD + lane * DPL + q] = acc2[rp][q].y;
+    }
   __syncthreads();
   for (int i = t; i < R * HD; i += kAttnThreads) {
     const int r = i / HD, dd = i - r * HD;

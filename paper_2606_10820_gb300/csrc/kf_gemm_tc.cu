@@ -183,8 +183,9 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   constexpr uint32_t A_BYTES = kBM * kBK * 2;
   constexpr uint32_t B_BYTES = BN * kBK * 2;
   constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static_assert(4 * 32 * 68 * 4 <= STAGES * STAGE_BYTES && kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
-                "epilogue blocks and split partials live in the idle pipeline stages");
+  static_assert(4 * 32 * 68 * 4 + kBM * 4 <= STAGES * STAGE_BYTES &&
+                    kBM * (BN + 4) * 4 + kBM * 4 <= STAGES * STAGE_BYTES,
+                "epilogue blocks, split partials and row scales live in the idle pipeline stages");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment for the 128B swizzle pattern
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -192,6 +193,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   // bars[0..S): full, bars[S..2S): empty, bars[2S]: accumulator ready
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
+  // fused-RMSNorm row scales: the last 512 bytes of the (then idle) stages
+  float* s_rinv = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES) - kBM;
   int* s_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -283,6 +286,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const int rbase = m0 + quarter * 32;
     const bool active = rbase < g.M;          // warp-uniform
+    if (ready && (EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in) {
+      // fused RMSNorm: the tile's 128 row scales, one row per epilogue thread
+      // (ready is uniform over the epilogue warps)
+      s_rinv[et] = (m0 + et < g.M) ? row_rinv(g.epi, m0 + et) : 0.f;
+      epi_bar();
+    }
     if (ready && active) {
       if (g.splits > 1) {
         // this split's partial: rows of the tile in the CTA's own shared
@@ -328,14 +337,31 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int row = rbase + gr + 4 * i;
-            const float4 lo = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + gc);
-            const float4 hi = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + 32 + gc);
-            if (row < g.M) {
+            const bool ok = row < g.M;                 // uniform over 8 lanes
+            float4 lo = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + gc);
+            float4 hi = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + 32 + gc);
+            if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && ok && g.epi.ss_in) {
+              const float r = s_rinv[row - m0];      // fused RMSNorm of the A rows
+              lo = scale4(lo, r);
+              hi = scale4(hi, r);
+            }
+            float sq = 0.f;
+            if (ok) {
               if (EPI == EPI_QKV) {
                 epi_qkv<__nv_bfloat16>(g.epi, row, n0 + c, gc, lo, hi);
               } else {
-                epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N);
-                epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
+                sq = epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N) +
+                     epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
+              }
+            }
+            if ((EPI == EPI_RESID || EPI == EPI_NOISE_OUT) && g.epi.ss_out) {
+              // the 8 lanes of this row hold its 64-column slot: fixed-order butterfly
+              sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+              sq += __shfl_xor_sync(0xffffffffu, sq, 2);
+              sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+              if (ok && (lane & 7) == 0) {
+                const int xr = (EPI == EPI_NOISE_OUT) ? g.epi.row_map[row] : row;
+                g.epi.ss_out[(size_t)xr * g.epi.nslot + (n0 + c) / 64] = sq;
               }
             }
           }
@@ -362,23 +388,26 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       const int rows_mine = (kBM - q + S - 1) / S;
       const int items = rows_mine * GROUPS;
       const uint32_t pbase = smem_u32(smem);
-      for (int it0 = et; it0 < items; it0 += 128 * U) {
+      // warp-uniform trip count (the butterflies below need every lane)
+      for (int it0 = et - (et & 31); it0 < items; it0 += 128 * U) {
         float4 acc[U];
         int row[U], gcol[U];
+        bool ok[U];
         uint32_t off[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-          const int idx = it0 + u * 128;
+          const int idx = it0 + (et & 31) + u * 128;
           const int rr = q + S * (idx / GROUPS);
           gcol[u] = (idx % GROUPS) * 4;
-          row[u] = (idx < items) ? m0 + rr : g.M;   // g.M marks "no item"
+          row[u] = m0 + rr;
+          ok[u] = idx < items && row[u] < g.M;
           off[u] = (uint32_t)((rr * (BN + 4) + gcol[u]) * 4);
           acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
         for (int sp = 0; sp < S; ++sp) {
 #pragma unroll
           for (int u = 0; u < U; ++u) {
-            if (row[u] < g.M) {
+            if (ok[u]) {
               const float4 v = ld_dsmem4(pbase + off[u], (uint32_t)sp);
               acc[u].x += v.x; acc[u].y += v.y; acc[u].z += v.z; acc[u].w += v.w;
             }
@@ -386,8 +415,21 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         }
         if (EPI != EPI_HEAD && EPI != EPI_QKV) {   // never split (host guarantees)
 #pragma unroll
-          for (int u = 0; u < U; ++u)
-            if (row[u] < g.M) epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N);
+          for (int u = 0; u < U; ++u) {
+            if (EPI == EPI_BIAS_GELU && ok[u] && g.epi.ss_in) acc[u] = scale4(acc[u], s_rinv[row[u] - m0]);
+            float sq = ok[u] ? epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N) : 0.f;
+            if ((EPI == EPI_RESID || EPI == EPI_NOISE_OUT) && g.epi.ss_out) {
+              // 16 consecutive lanes hold one row's 64-column slot
+              sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+              sq += __shfl_xor_sync(0xffffffffu, sq, 2);
+              sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+              sq += __shfl_xor_sync(0xffffffffu, sq, 8);
+              if (ok[u] && (et & 15) == 0) {
+                const int xr = (EPI == EPI_NOISE_OUT) ? g.epi.row_map[row[u]] : row[u];
+                g.epi.ss_out[(size_t)xr * g.epi.nslot + (n0 + gcol[u]) / 64] = sq;
+              }
+            }
+          }
         }
       }
     }

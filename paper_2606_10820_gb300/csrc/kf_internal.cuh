@@ -88,7 +88,26 @@ struct Epi {
   const float* cos_t = nullptr;    // [max_len][32] or NULL (no rotation)
   const float* sin_t = nullptr;
   int* d_err = nullptr;
+  // fused RMSNorm (tensor-core path).  Producers of the residual stream
+  // (EPI_RESID, EPI_NOISE_OUT) also write xb = bf16(x) and, per row, the sum
+  // of squares of each 64-column slot of x into ss_out[row][nslot].  The
+  // consumers (EPI_QKV, EPI_BIAS_GELU on the normed input) read ss_in and
+  // scale each row of D by rsqrt(sum / d + eps) (the gains are folded into
+  // their weights).
+  void* xb_out = nullptr;
+  float* ss_out = nullptr;
+  const float* ss_in = nullptr;
+  int nslot = 0;
+  float inv_d = 0.f, eps = 0.f;
 };
+
+// rsqrt(mean of squares + eps) of row `row` from its per-slot sums
+__device__ __forceinline__ float row_rinv(const Epi& e, int row) {
+  const float* p = e.ss_in + (size_t)row * e.nslot;
+  float s = 0.f;
+  for (int i = 0; i < e.nslot; ++i) s += p[i];
+  return rsqrtf(s * e.inv_d + e.eps);
+}
 
 // EPI_QKV for one row: lo = columns col0+gc .. +3 and hi = the same columns
 // + 32 of one 64-wide head block (col0 % 64 == 0, head_dim 64).  Rotates
@@ -215,8 +234,8 @@ __device__ __forceinline__ void st_ta4(__nv_bfloat16* p, float4 v) {
 }
 
 template <typename TA, int EPI>
-__device__ __forceinline__ void epi_vec4(const Epi& e, int row, int col, float4 v, int N) {
-  if (col >= N) return;
+__device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4 v, int N) {
+  if (col >= N) return 0.f;
   if (EPI == EPI_STORE) {
     st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
   } else if (EPI == EPI_STORE_F32) {
@@ -228,21 +247,25 @@ __device__ __forceinline__ void epi_vec4(const Epi& e, int row, int col, float4 
     }
     v = make_float4(gelu_tanh(v.x), gelu_tanh(v.y), gelu_tanh(v.z), gelu_tanh(v.w));
     st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
-  } else if (EPI == EPI_RESID) {
-    float4* p = reinterpret_cast<float4*>(e.x + (size_t)row * e.ldx + col);
-    float4 x = *p;
-    *p = make_float4(x.x + v.x, x.y + v.y, x.z + v.z, x.w + v.w);
-  } else if (EPI == EPI_NOISE_OUT) {
-    const int xr = e.row_map[row];
-    if (e.bias) {
-      float4 b = *reinterpret_cast<const float4*>(e.bias + col);
-      v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
-    }
-    if (e.pos_emb) {
-      float4 q = *reinterpret_cast<const float4*>(e.pos_emb + (size_t)e.row_pos[xr] * N + col);
-      v.x += q.x; v.y += q.y; v.z += q.z; v.w += q.w;
+  } else if (EPI == EPI_RESID || EPI == EPI_NOISE_OUT) {
+    int xr = row;
+    if (EPI == EPI_RESID) {
+      float4 x = *reinterpret_cast<const float4*>(e.x + (size_t)row * e.ldx + col);
+      v = make_float4(x.x + v.x, x.y + v.y, x.z + v.z, x.w + v.w);
+    } else {
+      xr = e.row_map[row];
+      if (e.bias) {
+        float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+        v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+      }
+      if (e.pos_emb) {
+        float4 q = *reinterpret_cast<const float4*>(e.pos_emb + (size_t)e.row_pos[xr] * N + col);
+        v.x += q.x; v.y += q.y; v.z += q.z; v.w += q.w;
+      }
     }
     *reinterpret_cast<float4*>(e.x + (size_t)xr * e.ldx + col) = v;
+    if (e.xb_out) st_ta4(reinterpret_cast<TA*>(e.xb_out) + (size_t)xr * e.ldx + col, v);
+    return v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   } else if (EPI == EPI_LOGITS) {
     float* o = e.outf + (size_t)row * e.ldo + col;
     const float t = e.inv_tau;
@@ -254,6 +277,11 @@ __device__ __forceinline__ void epi_vec4(const Epi& e, int row, int col, float4 
       if (col + 2 < e.n_valid) o[2] = v.z * t;
     }
   }
+  return 0.f;
+}
+
+__device__ __forceinline__ float4 scale4(float4 v, float r) {
+  return make_float4(v.x * r, v.y * r, v.z * r, v.w * r);
 }
 
 // ---------------------------------------------------------------- launches
@@ -332,12 +360,15 @@ void set_global_error(const std::string& msg);
 // elementwise / bookkeeping kernels
 void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
                    int32_t* noise_map, int32_t* head_map, cudaStream_t s);
+// xb / ss: bf16 copy and per-64-column sums of squares (fused RMSNorm), or NULL
 void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
                           const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
-                          int V, int d, float* x, int* d_err, cudaStream_t s);
+                          int V, int d, float* x, void* xb, float* ss, int* d_err, cudaStream_t s);
 void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
                          const float* pos_emb, const int32_t* row_pos, int V, int d, float* x,
-                         int* d_err, cudaStream_t s);
+                         void* xb, float* ss, int* d_err, cudaStream_t s);
+void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, size_t total,
+                       cudaStream_t s);
 void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
                        float scale, int d, void* feat, cudaStream_t s);
 void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,

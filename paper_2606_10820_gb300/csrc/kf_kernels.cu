@@ -36,64 +36,108 @@ void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, 
 }
 
 // ------------------------------------------------------------ embeddings
+// x[r] = E[tok] (+ pos_emb[pos]).  With the fused RMSNorm (xb != NULL) the
+// row is also written as bf16 into xb and the sum of squares of each of its
+// 64-column slots into ss[r][d/64] (warp partials over 32 columns, then the
+// pair of a slot added in order).
 template <typename TA>
 __device__ void embed_row(int r, int tok, int pos, const TA* __restrict__ emb,
-                          const float* __restrict__ pos_emb, int V, int d, float* x, int* d_err) {
+                          const float* __restrict__ pos_emb, int V, int d, float* x, TA* xb,
+                          float* ss, int* d_err) {
+  __shared__ float part[128];          // d <= 4096
   float* o = x + (size_t)r * d;
-  if (tok < 0 || tok >= V) {
-    if (threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
-    for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = 0.f;
-    return;
-  }
-  const TA* e = emb + (size_t)tok * d;
+  const bool good = tok >= 0 && tok < V;
+  if (!good && threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
+  const TA* e = emb + (size_t)(good ? tok : 0) * d;
   const float* p = pos_emb ? pos_emb + (size_t)pos * d : nullptr;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = to_f(e[c]) + (p ? p[c] : 0.f);
+  const int lane = threadIdx.x & 31;
+  for (int c0 = threadIdx.x - lane; c0 < d; c0 += blockDim.x) {
+    const int c = c0 + lane;
+    float v = 0.f;
+    if (c < d) {
+      v = good ? to_f(e[c]) + (p ? p[c] : 0.f) : 0.f;
+      o[c] = v;
+      if (xb) xb[(size_t)r * d + c] = from_f<TA>(v);
+    }
+    if (ss) {
+      float q = v * v;
+      for (int k = 16; k > 0; k >>= 1) q += __shfl_xor_sync(0xffffffffu, q, k);
+      if (lane == 0) part[c0 / 32] = q;
+    }
+  }
+  if (ss) {
+    __syncthreads();
+    for (int sl = threadIdx.x; sl < d / 64; sl += blockDim.x)
+      ss[(size_t)r * (d / 64) + sl] = part[2 * sl] + part[2 * sl + 1];
+  }
 }
 
 template <typename TA>
 __global__ void k_embed_pending(int P, int k, const int32_t* __restrict__ pending, int pend_stride,
                                 const TA* __restrict__ emb, const float* __restrict__ pos_emb,
                                 const int32_t* __restrict__ row_pos, int V, int d, float* x,
-                                int* d_err) {
+                                TA* xb, float* ss, int* d_err) {
   pdl_trigger();
   pdl_wait();
   int b = blockIdx.x / P, i = blockIdx.x - b * P;
   int r = b * (P + k) + i;
-  embed_row<TA>(r, pending[b * pend_stride + i], row_pos[r], emb, pos_emb, V, d, x, d_err);
+  embed_row<TA>(r, pending[b * pend_stride + i], row_pos[r], emb, pos_emb, V, d, x, xb, ss, d_err);
 }
 
 template <typename TA>
 __global__ void k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
                                const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
-                               int V, int d, float* x, int* d_err) {
+                               int V, int d, float* x, TA* xb, float* ss, int* d_err) {
   pdl_trigger();
   pdl_wait();
   int r = blockIdx.x;
-  embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, d_err);
+  embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, xb, ss, d_err);
 }
 
 void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
                           const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
-                          int V, int d, float* x, int* d_err, cudaStream_t s) {
+                          int V, int d, float* x, void* xb, float* ss, int* d_err, cudaStream_t s) {
   if (B * P == 0) return;
   if (bf16)
-    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(128), 0, s, P, k, pending, pend_stride,
-        (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
+    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(128), 0, s, P, k, pending,
+              pend_stride, (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x,
+              (__nv_bfloat16*)xb, ss, d_err);
   else
     kf_launch(k_embed_pending<float>, dim3(B * P), dim3(128), 0, s, P, k, pending, pend_stride,
-        (const float*)tok_emb, pos_emb, row_pos, V, d, x, d_err);
+              (const float*)tok_emb, pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
 }
 
 void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
                          const float* pos_emb, const int32_t* row_pos, int V, int d, float* x,
-                         int* d_err, cudaStream_t s) {
+                         void* xb, float* ss, int* d_err, cudaStream_t s) {
   if (R == 0) return;
   if (bf16)
-    kf_launch(k_embed_tokens<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_tok, (const __nv_bfloat16*)tok_emb,
-                                                    pos_emb, row_pos, V, d, x, d_err);
+    kf_launch(k_embed_tokens<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_tok,
+              (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x, (__nv_bfloat16*)xb, ss,
+              d_err);
   else
-    kf_launch(k_embed_tokens<float>, dim3(R), dim3(128), 0, s, row_tok, (const float*)tok_emb, pos_emb, row_pos, V,
-                                            d, x, d_err);
+    kf_launch(k_embed_tokens<float>, dim3(R), dim3(128), 0, s, row_tok, (const float*)tok_emb,
+              pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
+}
+
+// w[r][c] *= g[(r / rows_per_layer) * cols + c]: folds RMSNorm gains into the
+// columns of the projection that consumes the normed rows
+__global__ void k_scale_cols(float* __restrict__ w, const float* __restrict__ g, int rows_per_layer,
+                             int cols, size_t total) {
+  size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  size_t stride = (size_t)gridDim.x * blockDim.x;
+  for (; i < total; i += stride) {
+    const size_t r = i / cols;
+    const int c = (int)(i - r * cols);
+    w[i] *= g[(r / rows_per_layer) * cols + c];
+  }
+}
+
+void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, size_t total,
+                       cudaStream_t s) {
+  if (total == 0) return;
+  int blocks = (int)std::min<size_t>((total + 255) / 256, 65535);
+  k_scale_cols<<<blocks, 256, 0, s>>>(w, g, rows_per_layer, cols, total);
 }
 
 // ------------------------------------------------------- noise features

@@ -158,6 +158,21 @@ def test_pdl_equals_plain_launches(kf):
             np.testing.assert_array_equal(a, b)
 
 
+def test_norm_gains_folded(kf):
+    """Non-unit RMSNorm gains: the fused path folds them into the QKV and
+    MLP-up weights; the oracle applies them after normalising."""
+    cfg = LM1B.replace(n_layer=2)
+    w = make_weights(cfg)
+    rng = np.random.default_rng(9)
+    for name in ("attn_norm", "mlp_norm", "final_norm"):
+        w[name] = (1.0 + 0.3 * rng.standard_normal(w[name].shape)).astype(np.float32)
+    prompts = make_prompts([20, 31], cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 0, 2], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
+
+
 def test_device_buffers(kf):
     import torch
     cfg = TINY
