@@ -45,6 +45,9 @@ def parse():
     p.add_argument("--gen", type=int, default=0, help="tokens per sequence (0: workload)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--no-ar", action="store_true", help="skip the k=1 AR leg")
+    p.add_argument("--sweep", action="store_true",
+                   help="one line per configuration: OWT-shaped batch 1..256, OWT paged "
+                        "batch 512, medium batch 256 (k vs the AR step)")
     return p.parse_args()
 
 
@@ -55,6 +58,17 @@ def peaks():
             d = json.load(f)
         return d, "measured"
     return FALLBACK_PEAKS, "fallback"
+
+
+def max_over_ranks(x: float, dist) -> float:
+    """Largest value of x over all ranks (the slowest rank's time)."""
+    if dist is None:
+        return x
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
 
 
 def dist_init(n):
@@ -208,18 +222,18 @@ def run_reference(args):
     w, B, gen = workload_of(args)
     model = w.model
     weights = make_weights(model)
-    Bs = min(B, 4)
+    Bs = min(B, 16)
     prompts = workload_prompts(w, Bs)
     rates = []
     for _ in range(max(1, args.warmup and 1)):
         cpu_oracle_rate(model, weights, prompts, args.k, budget_s=5.0, max_calls=2)
     t_all = time.perf_counter()
     for _ in range(args.steps):
-        r, calls, el = cpu_oracle_rate(model, weights, prompts, args.k, budget_s=20.0, max_calls=3)
+        r, calls, el = cpu_oracle_rate(model, weights, prompts, args.k, budget_s=10.0, max_calls=24)
         rates.append(r)
     el = time.perf_counter() - t_all
     v = statistics.median(rates)
-    sample = f"{Bs} sequences x up to 3 decode calls of k={args.k} per step (prompt {w.prompt_len})"
+    sample = f"{Bs} sequences x decode calls of k={args.k} for up to 10 s per step (prompt {w.prompt_len})"
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000 * el / max(1, args.steps), "higher_is_better": True,
@@ -233,8 +247,93 @@ def run_reference(args):
     return 0
 
 
+SWEEP = [  # (workload, batch, ks) -- the non-headline configurations
+    ("owt", 1, (4, 2, 1)), ("owt", 8, (4, 2, 1)), ("owt", 32, (4, 2, 1)),
+    ("owt", 128, (4, 2, 1)), ("owt", 256, (4, 2, 1)),
+    ("owt_paged", 512, (4, 1)),
+    ("medium", 256, (8, 4, 1)),
+]
+
+
+def run_sweep(args):
+    """Tokens/s of full generations per configuration, k vs the AR step, with
+    the step roofline fraction; one JSON line each (rank 0, N = 1)."""
+    import torch
+    from paper_2606_10820_gb300 import build as kbuild
+    from paper_2606_10820_gb300 import kforcing as kf
+    from synth import WORKLOADS, make_weights, workload_prompts
+    kbuild.build()
+    kf.load_library()
+    pk, peak_src = peaks()
+    by_wl = {}
+    for name, B, ks in SWEEP:
+        by_wl.setdefault(name, []).append((B, ks))
+    for name, runs in by_wl.items():
+        w = WORKLOADS[name]
+        model = w.model
+        weights = make_weights(model)
+        maxB = max(B for B, _ in runs)
+        maxk = max(max(ks) for _, ks in runs)
+        stream = torch.cuda.Stream()
+        dec = kf.Decoder(model, weights, max_batch=maxB, max_k=maxk, stream=stream.cuda_stream)
+        del weights
+        for B, ks in runs:
+            prompts = workload_prompts(w, B)
+            dec.prefill(prompts)
+            gen = w.gen_len
+            res = {}
+            for k in ks:
+                kk = 0 if k == 1 else k          # k=1 is the AR teacher step
+                nout = max(kk, 1)
+                calls = -(-gen // nout)
+                z = torch.rand((calls, B, nout), device="cuda")
+                o = torch.zeros((calls, B, nout), dtype=torch.int32, device="cuda")
+
+                def one():
+                    dec.rewind()
+                    for i in range(calls):
+                        kf.kf_decode_step(dec.ctx, B, kk, z[i], o[i])
+                for _ in range(max(1, args.warmup)):
+                    one()
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for _ in range(args.steps):
+                    one()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                ms = e0.elapsed_time(e1) / args.steps
+                t_roof = 0.0
+                for i in range(calls):
+                    P = 1 if i == 0 else nout
+                    lens = np.array([len(p) - 1 + (0 if i == 0 else 1 + (i - 1) * nout) for p in prompts])
+                    byt, fl = step_bytes_flops(model, B, P, kk, lens)
+                    t_roof += max(byt / (pk["hbm_gbs"] * 1e9), fl / (pk["bf16_tflops_sustained"] * 1e12))
+                res[k] = {"value": B * calls * nout / (ms / 1e3), "ms_per_step": ms,
+                          "step_roofline_frac": t_roof * 1e3 / ms}
+            kmax = max(ks)
+            line = {"metric": METRIC, "value": res[kmax]["value"], "unit": "tokens/s", "n_gpus": 1,
+                    "steps": args.steps, "warmup": args.warmup,
+                    "ms_per_step": res[kmax]["ms_per_step"], "higher_is_better": True,
+                    "scaling": "weak", "vs_baseline": None, "dtype": model.dtype,
+                    "data": "synthetic", "sweep": True,
+                    "config": {"workload": f"{name}: {model.n_layer}L d{model.d_model} V{model.vocab}, "
+                                           f"batch {B}, prompt {w.prompt_len or list(w.ragged)} +{gen}",
+                               "batch": B, "k": kmax},
+                    "per_k": {str(k): {kk_: round(v, 4) for kk_, v in r.items()} for k, r in res.items()},
+                    "speedup_vs_k1": {str(k): res[k]["value"] / res[1]["value"] for k in ks if 1 in res},
+                    "peak_source": peak_src}
+            print(json.dumps(line), flush=True)
+        dec.close()
+        del dec
+        torch.cuda.empty_cache()
+    return 0
+
+
 def main():
     args = parse()
+    if args.sweep:
+        return run_sweep(args)
     if args.impl == "reference":
         return run_reference(args)
     import torch
@@ -294,10 +393,7 @@ def main():
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
         ms = e0.elapsed_time(e1) if not host else wall * 1000.0
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
+        ms = max_over_ranks(ms, dist)
         tokens = world * args.steps * B * calls * nout
         return tokens / (ms / 1000.0), ms / args.steps, calls, z.nbytes // calls * calls
 
@@ -366,9 +462,9 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu:
-        Bs = min(B, 4)
+        Bs = min(B, 16)
         r, ncalls, el = cpu_oracle_rate(model, weights, prompts[:Bs], k, budget_s=15.0,
-                                        max_calls=3)
+                                        max_calls=24)
         cpu = {"value": r, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
                "sample": f"{Bs} of the {B} sequences, {ncalls} decode calls of k={k} "
                          f"after the prompt ({el:.1f} s, numpy fp64)"}

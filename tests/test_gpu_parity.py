@@ -10,7 +10,8 @@ import numpy as np
 import pytest
 
 import oracle
-from synth import LM1B, OWT, TINY, make_noise, make_prompt_lengths, make_prompts, make_weights
+from synth import (LM1B, MEDIUM, OWT, TINY, WORKLOADS, make_noise, make_prompt_lengths,
+                   make_prompts, make_weights, workload_prompts)
 
 from parity import LOGIT_TOL, compare_tokens, logit_check
 
@@ -301,3 +302,50 @@ def test_owt_ragged_paged(kf):
     worst, slots, mism, bad = _bf16_check(recs)
     assert worst <= LOGIT_TOL and bad == 0
     dec.close()
+
+
+def _sampled(kf, cfg, w, prompts, pick, ks, max_k, seed):
+    """Full batch on the GPU (graph replay), the oracle on sampled sequences."""
+    B = len(prompts)
+    dec = kf.Decoder(cfg, w, max_batch=B, max_k=max_k)
+    dec.prefill(prompts)
+    ref = oracle.OracleDecoder(oracle.OracleModel(cfg, w))
+    ref.prefill([prompts[i] for i in pick])
+    rng = np.random.default_rng(seed)
+    worst, slots, mism, bad = 0.0, 0, 0, 0
+    for k in ks:
+        z = rng.random((B, max(k, 1)), dtype=np.float32)
+        gt = dec.step(k, z)
+        gl = dec.logits(max(k, 1))[pick]
+        rt, rl = ref.step(k, z[pick], want_logits=True)
+        worst = max(worst, logit_check(gl, rl))
+        n, m, u = compare_tokens(gt[pick], rt, gl, rl, z[pick])
+        slots, mism, bad = slots + n, mism + m, bad + u
+        for j, b in enumerate(pick):
+            ref.seqs[j]["pending"] = [int(t) for t in gt[b]]
+        assert [int(x) for x in dec.lengths()[pick]] == [ref.cached_len(j) for j in range(len(pick))]
+    dec.close()
+    return worst, slots, mism, bad
+
+
+def test_owt_paged_full_batch_sampled(kf):
+    """OWT-shaped high-load serving: batch 512, ragged prompts in [128, 896],
+    16-token pages; sampled sequences against the oracle."""
+    wl = WORKLOADS["owt_paged"]
+    cfg = wl.model
+    w = make_weights(cfg)
+    prompts = workload_prompts(wl)
+    lens = [len(p) for p in prompts]
+    pick = [int(np.argmin(lens)), int(np.argmax(lens)), 100, 511]
+    worst, slots, mism, bad = _sampled(kf, cfg, w, prompts, pick, [4, 4, 0], 4, 21)
+    assert worst <= LOGIT_TOL and bad == 0
+
+
+def test_medium_k8_sampled(kf):
+    """Medium stress shape (24 layers, d 1024, 16 heads): batch 256, prompts
+    of 1024, k = 8 then k = 4; sampled sequences against the oracle."""
+    cfg = MEDIUM
+    w = make_weights(cfg)
+    prompts = make_prompts([1024] * 256, cfg.vocab)
+    worst, slots, mism, bad = _sampled(kf, cfg, w, prompts, [0, 255], [8, 8, 4], 8, 22)
+    assert worst <= LOGIT_TOL and bad == 0
