@@ -186,12 +186,15 @@ static void gemm(kf_ctx* c, int kind, int M, int N, int K, const void* A, int ld
   prof_end(c);
 }
 
-// attention split count: enough CTAs to cover the SMs twice
-static void attn_plan(kf_ctx* c, int n_groups, int R, int* n_split, int* kps) {
+// attention split count: enough CTAs to cover the SMs twice, and at most
+// max_keys keys per CTA
+static void attn_plan(kf_ctx* c, int n_groups, int R, int max_keys, int* n_split, int* kps) {
   int ctas = n_groups * c->H;
   int max_split = ceil_div(c->cfg.max_len, 64);
   int s = std::max(1, std::min(max_split, ceil_div(2 * c->num_sms, std::max(1, ctas))));
-  while (s > 1 && (size_t)s * R * c->H > c->part_units) --s;
+  s = std::max(s, ceil_div(c->cfg.max_len, max_keys));
+  while (s > 1 && (size_t)s * R * c->H > c->part_units && ceil_div(c->cfg.max_len, s - 1) <= max_keys)
+    --s;
   *n_split = s;
   *kps = round_up(ceil_div(c->cfg.max_len, s), 64);
 }
@@ -205,8 +208,14 @@ static void attn_plan(kf_ctx* c, int n_groups, int R, int* n_split, int* kps) {
 static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, int uniform_rows) {
   const int d = c->d, H = c->H, F = c->F;
   cudaStream_t s = c->stream;
+  // Tensor-core attention on the fused bf16 path for groups of more than 8
+  // query rows (k = 8 steps, prefill); with 1..8 rows its per-tile MMA round
+  // trips and V transpose cost more than FMA scores (measured), so those use
+  // the CUDA-core kernel.
+  const int rows = groups ? kMaxGroupRows : uniform_rows;
+  const bool tc_attn = c->fused && rows > 8;
   int n_split, kps;
-  attn_plan(c, n_groups, R, &n_split, &kps);
+  attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
   auto norm_in = [&](Epi& e) {
     e.ss_in = c->ss; e.nslot = d / 64; e.inv_d = 1.0f / d; e.eps = c->cfg.rms_eps;
   };
@@ -246,7 +255,8 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     prof_begin(c, KF_KIND_ATTENTION);
-    launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
+    if (tc_attn) launch_attention_tc(a, n_groups, s);
+    else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
     if (n_split > 1) {
       prof_begin(c, KF_KIND_ATTN_COMBINE);
@@ -541,7 +551,12 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
       (r = dalloc(c, &c->head_map, (size_t)c->NR_cap * 4)) ||
       (r = dalloc(c, &c->groups, (size_t)R * sizeof(int4))) || (r = dalloc(c, &c->d_err, 4)))
     return bail(r);
+  // split-KV partials: small batches split to fill the SMs; the tensor-core
+  // attention also splits every context longer than its per-CTA key limit
   c->part_units = (size_t)4 * c->num_sms * kMaxGroupRows;
+  if (c->fused)
+    c->part_units = std::max(c->part_units, (size_t)ceil_div(cfg.max_len, attention_tc_max_keys()) *
+                                                c->R_cap * c->H);
   if ((r = dalloc(c, &c->part_o, c->part_units * c->hd * 4)) ||
       (r = dalloc(c, &c->part_ml, c->part_units * sizeof(float2))))
     return bail(r);

@@ -353,6 +353,10 @@ struct AttnArgs {
 // max_keys: the most keys any row of the launch can see (max_len bound)
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
 void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
+// tensor-core decode attention (bf16 cache, head_dim 64, <= 16 rows per group,
+// keys_per_split <= attention_tc_max_keys())
+void launch_attention_tc(const AttnArgs& a, int n_groups, cudaStream_t s);
+int attention_tc_max_keys();
 
 // message for kf_last_error(NULL) (calls without a context)
 void set_global_error(const std::string& msg);
