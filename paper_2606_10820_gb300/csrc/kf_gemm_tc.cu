@@ -9,8 +9,12 @@
 //   warp 1      allocates TMEM; one lane issues tcgen05.mma and commits each
 //               stage back to the producer and the finished tile to the
 //               epilogue;
-//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns per warp (one
-//               output row's run of 32 columns per thread) -> epi_run32.
+//   warps 2..9  epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31 (its 32
+//               rows); the two warps of a lane quarter take alternate
+//               64-column blocks of the tile (or, with a single block,
+//               alternate halves of its rows).  While the mainloop runs they
+//               fetch the per-row data of the tile (RMSNorm scales, positions,
+//               KV pages) into shared memory.
 // When the output tiles cannot fill the SMs the K range is split over a
 // thread-block cluster of up to 8 CTAs (one per split): each keeps its fp32
 // partial tile in its own shared memory and, after a cluster barrier, CTA q
@@ -32,7 +36,15 @@ namespace kf {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;                 // one 128-byte swizzle atom of bf16
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + 32 * kEpiWarps;
+
+// per-row data of a tile, fetched by the epilogue warps during the mainloop
+struct EpiMeta {
+  float rinv[kBM];   // fused RMSNorm scale of the A row
+  int pos[kBM];      // EPI_QKV: position of the row
+  int aux[kBM];      // EPI_QKV: KV page of the row (-1 if invalid)
+};
 
 struct TcArgs {
   int M, N, K;
@@ -43,7 +55,7 @@ struct TcArgs {
 };
 
 __device__ __forceinline__ void epi_bar() {
-  asm volatile("bar.sync 1, 128;" ::: "memory");
+  asm volatile("bar.sync 1, %0;" ::"n"(32 * kEpiWarps) : "memory");
 }
 
 // ------------------------------------------------------------ the kernel
@@ -54,9 +66,9 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   constexpr uint32_t A_BYTES = kBM * kBK * 2;
   constexpr uint32_t B_BYTES = BN * kBK * 2;
   constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static_assert(4 * 32 * 68 * 4 + kBM * 4 <= STAGES * STAGE_BYTES &&
-                    kBM * (BN + 4) * 4 + kBM * 4 <= STAGES * STAGE_BYTES,
-                "epilogue blocks, split partials and row scales live in the idle pipeline stages");
+  static_assert(kEpiWarps * 32 * 68 * 4 <= STAGES * STAGE_BYTES &&
+                    kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
+                "epilogue blocks and split partials live in the idle pipeline stages");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment for the 128B swizzle pattern
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -64,9 +76,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   // bars[0..S): full, bars[S..2S): empty, bars[2S]: accumulator ready
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
-  // fused-RMSNorm row scales: the last 512 bytes of the (then idle) stages
-  float* s_rinv = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES) - kBM;
   int* s_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  EpiMeta* meta = reinterpret_cast<EpiMeta*>(smem + STAGES * STAGE_BYTES + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_tile = blockIdx.x, m_tile = blockIdx.y, split = blockIdx.z;
@@ -145,10 +156,33 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       if (ok) mma_commit(smem_u32(&bars[2 * STAGES]));
     }
   } else {
-    // epilogue warps 2..5: TMEM lanes 32*(warp%4) .. +31
-    const int quarter = warp & 3;
-    const int et = threadIdx.x - 64;              // 0..127
+    const int quarter = warp & 3;                 // TMEM lanes 32*quarter .. +31
+    const int ch = (warp - 2) >> 2;               // which warp of the quarter
+    const int et = threadIdx.x - 64;              // 0 .. 32*kEpiWarps-1
     pdl_wait();
+    // the tile's per-row data, while the mainloop runs
+    if (et < kBM) {
+      const int row = m0 + et;
+      const bool in = row < g.M;
+      if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in)
+        meta->rinv[et] = in ? row_rinv(g.epi, row) : 0.f;
+      if (EPI == EPI_QKV) {
+        int pos = 0, page = -1;
+        if (in) {
+          pos = __ldg(g.epi.row_pos + row);
+          const int pi = pos / kPage;
+          page = pi < g.epi.max_pages
+                     ? __ldg(g.epi.page_table + (size_t)__ldg(g.epi.row_seq + row) * g.epi.max_pages + pi)
+                     : -1;
+          if (page < 0 || page >= g.epi.n_pages) {
+            page = -1;
+            atomicOr(g.epi.d_err, kErrBadPage);
+          }
+        }
+        meta->pos[et] = pos;
+        meta->aux[et] = page;
+      }
+    }
     // one waiter, result broadcast: every epilogue thread takes the same path
     if (et == 0) s_flag[1] = mbar_wait(smem_u32(&bars[2 * STAGES]), 0, g.d_err) ? 1 : 0;
     epi_bar();
@@ -157,19 +191,14 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const int rbase = m0 + quarter * 32;
     const bool active = rbase < g.M;          // warp-uniform
-    if (ready && (EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in) {
-      // fused RMSNorm: the tile's 128 row scales, one row per epilogue thread
-      // (ready is uniform over the epilogue warps)
-      s_rinv[et] = (m0 + et < g.M) ? row_rinv(g.epi, m0 + et) : 0.f;
-      epi_bar();
-    }
     if (ready && active) {
       if (g.splits > 1) {
         // this split's partial: rows of the tile in the CTA's own shared
-        // memory (pitch BN + 4), reduced across the cluster below
+        // memory (pitch BN + 4), reduced across the cluster below; the two
+        // warps of a quarter write alternate halves of the columns
         float* P = reinterpret_cast<float*>(smem) + (size_t)(quarter * 32 + lane) * (BN + 4);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = ch * (BN / 2); c < (ch + 1) * (BN / 2); c += 32) {
           float v[32];
           tmem_ld32(lane_addr + c, v);
 #pragma unroll
@@ -178,10 +207,11 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
                 make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
       } else if (EPI == EPI_HEAD) {
-        // row mode: a thread reduces its row's 32-id chunks
+        // row mode: a thread reduces its row's 32-id chunks (alternate
+        // halves of the tile's columns per warp of the quarter)
         const int row = rbase + lane;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = ch * (BN / 2); c < (ch + 1) * (BN / 2); c += 32) {
           float v[32];
           tmem_ld32(lane_addr + c, v);
           if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
@@ -191,10 +221,15 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         // tcgen05.ld gives a thread one row's columns; re-read with lane l on
         // row (l / 8) + 4 i, columns 4 (l % 8) .. +3 (and + 32): every warp
         // store covers four 128-byte row segments.
-        float* T = reinterpret_cast<float*>(smem) + quarter * (32 * 68);
+        constexpr int NB = BN / 64;                 // 64-column blocks
+        constexpr int NI = NB >= 2 ? 8 : 4;         // row groups per warp
+        const int b0 = NB >= 2 ? ch : 0;
+        const int ibase = NB >= 2 ? 0 : ch * 4;
+        float* T = reinterpret_cast<float*>(smem) + (warp - 2) * (32 * 68);
         const int gr = lane >> 3, gc = (lane & 7) * 4;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 64) {
+        for (int bb = b0; bb < NB; bb += (NB >= 2 ? 2 : 1)) {
+          const int c = bb * 64;
 #pragma unroll
           for (int h2 = 0; h2 < 2; ++h2) {
             float v[32];
@@ -206,20 +241,21 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
           }
           __syncwarp();
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int row = rbase + gr + 4 * i;
+          for (int ii = 0; ii < NI; ++ii) {
+            const int rl = quarter * 32 + gr + 4 * (ibase + ii);   // row within the tile
+            const int row = m0 + rl;
             const bool ok = row < g.M;                 // uniform over 8 lanes
-            float4 lo = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + gc);
-            float4 hi = *reinterpret_cast<const float4*>(T + (gr + 4 * i) * 68 + 32 + gc);
+            float4 lo = *reinterpret_cast<const float4*>(T + (rl - quarter * 32) * 68 + gc);
+            float4 hi = *reinterpret_cast<const float4*>(T + (rl - quarter * 32) * 68 + 32 + gc);
             if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && ok && g.epi.ss_in) {
-              const float r = s_rinv[row - m0];      // fused RMSNorm of the A rows
+              const float r = meta->rinv[rl];        // fused RMSNorm of the A rows
               lo = scale4(lo, r);
               hi = scale4(hi, r);
             }
             float sq = 0.f;
             if (ok) {
               if (EPI == EPI_QKV) {
-                epi_qkv<__nv_bfloat16>(g.epi, row, n0 + c, gc, lo, hi);
+                epi_qkv<__nv_bfloat16>(g.epi, row, meta->pos[rl], meta->aux[rl], n0 + c, gc, lo, hi);
               } else {
                 sq = epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N) +
                      epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
@@ -260,14 +296,14 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       const int items = rows_mine * GROUPS;
       const uint32_t pbase = smem_u32(smem);
       // warp-uniform trip count (the butterflies below need every lane)
-      for (int it0 = et - (et & 31); it0 < items; it0 += 128 * U) {
+      for (int it0 = et - (et & 31); it0 < items; it0 += 32 * kEpiWarps * U) {
         float4 acc[U];
         int row[U], gcol[U];
         bool ok[U];
         uint32_t off[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-          const int idx = it0 + (et & 31) + u * 128;
+          const int idx = it0 + (et & 31) + u * 32 * kEpiWarps;
           const int rr = q + S * (idx / GROUPS);
           gcol[u] = (idx % GROUPS) * 4;
           row[u] = m0 + rr;
@@ -287,7 +323,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         if (EPI != EPI_HEAD && EPI != EPI_QKV) {   // never split (host guarantees)
 #pragma unroll
           for (int u = 0; u < U; ++u) {
-            if (EPI == EPI_BIAS_GELU && ok[u] && g.epi.ss_in) acc[u] = scale4(acc[u], s_rinv[row[u] - m0]);
+            if (EPI == EPI_BIAS_GELU && ok[u] && g.epi.ss_in) acc[u] = scale4(acc[u], meta->rinv[row[u] - m0]);
             float sq = ok[u] ? epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N) : 0.f;
             if ((EPI == EPI_RESID || EPI == EPI_NOISE_OUT) && g.epi.ss_out) {
               // 16 consecutive lanes hold one row's 64-column slot
@@ -370,7 +406,7 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
     while (splits < 8 && tiles * splits * 2 <= num_sms && kb_total >= splits * 4) splits *= 2;
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
-  const size_t smem = (size_t)STAGES * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256;
+  const size_t smem = (size_t)STAGES * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,

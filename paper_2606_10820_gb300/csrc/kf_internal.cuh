@@ -39,6 +39,16 @@ __device__ __forceinline__ float gelu_tanh(float x) {
   const float c = 0.7978845608028654f;  // sqrt(2/pi)
   return 0.5f * x * (1.0f + tanhf(c * (x + 0.044715f * x * x * x)));
 }
+// the same with the hardware tanh (tanh.approx.f32, absolute error about
+// 5e-4): for bf16 outputs, whose rounding (2^-9 relative) is of that size
+__device__ __forceinline__ float gelu_tanh_bf16(float x) {
+  const float c = 0.7978845608028654f;
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(c * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.0f + t);
+}
+template <typename TA> __device__ __forceinline__ float gelu_for(float x) { return gelu_tanh(x); }
+template <> __device__ __forceinline__ float gelu_for<__nv_bfloat16>(float x) { return gelu_tanh_bf16(x); }
 
 // ---------------------------------------------------------------- GEMM epilogues
 // Every GEMM computes D[M][N] = A[M][K] . W[N][K]^T with fp32 accumulation and
@@ -109,19 +119,19 @@ __device__ __forceinline__ float row_rinv(const Epi& e, int row) {
   return rsqrtf(s * e.inv_d + e.eps);
 }
 
-// EPI_QKV for one row: lo = columns col0+gc .. +3 and hi = the same columns
-// + 32 of one 64-wide head block (col0 % 64 == 0, head_dim 64).  Rotates
-// the pairs (i, i + 32) of q and k at the row's position and stores q, k, v.
+// EPI_QKV for one row at position pos whose KV page is `page` (-1: invalid,
+// already flagged): lo = columns col0+gc .. +3 and hi = the same columns + 32
+// of one 64-wide head block (col0 % 64 == 0, head_dim 64).  Rotates the
+// pairs (i, i + 32) of q and k at the row's position and stores q, k, v.
 template <typename TA>
-__device__ __forceinline__ void epi_qkv(const Epi& e, int row, int col0, int gc, float4 lo,
-                                        float4 hi) {
+__device__ __forceinline__ void epi_qkv(const Epi& e, int row, int pos, int page, int col0, int gc,
+                                        float4 lo, float4 hi) {
   const int sec = col0 / e.dsec;                 // 0 q, 1 k, 2 v
   const int h = (col0 - sec * e.dsec) >> 6;
-  const int pos = e.row_pos[row];
   float a[4] = {lo.x, lo.y, lo.z, lo.w}, b[4] = {hi.x, hi.y, hi.z, hi.w};
   if (sec < 2 && e.cos_t) {
-    const float4 c4 = *reinterpret_cast<const float4*>(e.cos_t + (size_t)pos * 32 + gc);
-    const float4 s4 = *reinterpret_cast<const float4*>(e.sin_t + (size_t)pos * 32 + gc);
+    const float4 c4 = __ldg(reinterpret_cast<const float4*>(e.cos_t + (size_t)pos * 32 + gc));
+    const float4 s4 = __ldg(reinterpret_cast<const float4*>(e.sin_t + (size_t)pos * 32 + gc));
     const float c[4] = {c4.x, c4.y, c4.z, c4.w}, sn[4] = {s4.x, s4.y, s4.z, s4.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -136,13 +146,7 @@ __device__ __forceinline__ void epi_qkv(const Epi& e, int row, int col0, int gc,
     *reinterpret_cast<float4*>(q + 32) = make_float4(b[0], b[1], b[2], b[3]);
     return;
   }
-  const int bseq = e.row_seq[row];
-  const int pi = pos / kPage;
-  const int page = pi < e.max_pages ? e.page_table[bseq * e.max_pages + pi] : -1;
-  if (page < 0 || page >= e.n_pages) {
-    atomicOr(e.d_err, kErrBadPage);
-    return;
-  }
+  if (page < 0) return;
   TA* dst = reinterpret_cast<TA*>(e.kv) +
             ((((size_t)e.layer * e.n_pages + page) * 2 + (sec - 1)) * e.H + h) * (kPage * 64) +
             (size_t)(pos % kPage) * 64 + gc;
@@ -242,10 +246,10 @@ __device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4
     *reinterpret_cast<float4*>(e.outf + (size_t)row * e.ldo + col) = v;
   } else if (EPI == EPI_BIAS_GELU) {
     if (e.bias) {
-      float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+      float4 b = __ldg(reinterpret_cast<const float4*>(e.bias + col));
       v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
     }
-    v = make_float4(gelu_tanh(v.x), gelu_tanh(v.y), gelu_tanh(v.z), gelu_tanh(v.w));
+    v = make_float4(gelu_for<TA>(v.x), gelu_for<TA>(v.y), gelu_for<TA>(v.z), gelu_for<TA>(v.w));
     st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
   } else if (EPI == EPI_RESID || EPI == EPI_NOISE_OUT) {
     int xr = row;
@@ -255,11 +259,11 @@ __device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4
     } else {
       xr = e.row_map[row];
       if (e.bias) {
-        float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+        float4 b = __ldg(reinterpret_cast<const float4*>(e.bias + col));
         v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
       }
       if (e.pos_emb) {
-        float4 q = *reinterpret_cast<const float4*>(e.pos_emb + (size_t)e.row_pos[xr] * N + col);
+        float4 q = __ldg(reinterpret_cast<const float4*>(e.pos_emb + (size_t)e.row_pos[xr] * N + col));
         v.x += q.x; v.y += q.y; v.z += q.z; v.w += q.w;
       }
     }
