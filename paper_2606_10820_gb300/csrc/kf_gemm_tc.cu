@@ -36,6 +36,8 @@ namespace kf {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;                 // one 128-byte swizzle atom of bf16
+constexpr int kAtoms = 2;               // K atoms per pipeline stage (one wait and one
+                                        // commit per 8 MMAs)
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 
@@ -63,9 +65,10 @@ template <int BN, int STAGES, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
           TcArgs g) {
-  constexpr uint32_t A_BYTES = kBM * kBK * 2;
-  constexpr uint32_t B_BYTES = BN * kBK * 2;
-  constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr uint32_t A_ATOM = kBM * kBK * 2;            // one 128 x 64 A box
+  constexpr uint32_t B_ATOM = BN * kBK * 2;             // one BN x 64 W box
+  constexpr uint32_t A_BYTES = kAtoms * A_ATOM;
+  constexpr uint32_t STAGE_BYTES = kAtoms * (A_ATOM + B_ATOM);   // [A atoms][W atoms]
   static_assert(kEpiWarps * 32 * 68 * 4 <= STAGES * STAGE_BYTES &&
                     kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
                 "epilogue blocks and split partials live in the idle pipeline stages");
@@ -85,7 +88,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   const int kb_total = g.K / kBK;
   const int kb0 = split * g.kb_per_split;
   const int kb1 = min(kb_total, kb0 + g.kb_per_split);
-  const int nkb = kb1 - kb0;
+  const int nkb = kb1 - kb0;                  // K atoms of this split
+  const int nst = (nkb + kAtoms - 1) / kAtoms; // pipeline stages (the last may be short)
   pdl_trigger();
 
   if (threadIdx.x == 0) {
@@ -115,42 +119,58 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       // Weights are constant during a step: the first stages' weight tiles
       // stream in while the predecessor kernel finishes; the activation tiles
       // it produces are loaded after pdl_wait.
-      const int pre = min(nkb, STAGES);
+      const int pre = min(nst, STAGES);
       for (int i = 0; i < pre; ++i) {
         const uint32_t full = smem_u32(&bars[i]);
-        mbar_expect_tx(full, STAGE_BYTES);
-        tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES, &map_w, full, (kb0 + i) * kBK, n0);
+        const int na = min(kAtoms, nkb - i * kAtoms);
+        mbar_expect_tx(full, na * (A_ATOM + B_ATOM));
+        for (int a = 0; a < na; ++a)
+          tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES + a * B_ATOM, &map_w, full,
+                      (kb0 + i * kAtoms + a) * kBK, n0);
       }
       pdl_wait();
-      for (int i = 0; i < pre; ++i)
-        tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &map_a, smem_u32(&bars[i]), (kb0 + i) * kBK, m0);
-      for (int i = pre; i < nkb; ++i) {
+      for (int i = 0; i < pre; ++i) {
+        const int na = min(kAtoms, nkb - i * kAtoms);
+        for (int a = 0; a < na; ++a)
+          tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + a * A_ATOM, &map_a, smem_u32(&bars[i]),
+                      (kb0 + i * kAtoms + a) * kBK, m0);
+      }
+      for (int i = pre; i < nst; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (i / STAGES) & 1;
         if (!mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, g.d_err)) break;
         const uint32_t full = smem_u32(&bars[s]);
-        mbar_expect_tx(full, STAGE_BYTES);
+        const int na = min(kAtoms, nkb - i * kAtoms);
+        mbar_expect_tx(full, na * (A_ATOM + B_ATOM));
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
-        const int kc = (kb0 + i) * kBK;
-        tma_load_2d(sa, &map_a, full, kc, m0);
-        tma_load_2d(sa + A_BYTES, &map_w, full, kc, n0);
+        for (int a = 0; a < na; ++a) {
+          const int kc = (kb0 + i * kAtoms + a) * kBK;
+          tma_load_2d(sa + a * A_ATOM, &map_a, full, kc, m0);
+          tma_load_2d(sa + A_BYTES + a * B_ATOM, &map_w, full, kc, n0);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, BN);
       bool ok = true;
-      for (int i = 0; i < nkb; ++i) {
+      for (int i = 0; i < nst; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (i / STAGES) & 1;
         if (!mbar_wait(smem_u32(&bars[s]), ph, g.d_err)) { ok = false; break; }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
         const uint32_t sb = sa + A_BYTES;
+        const int na = min(kAtoms, nkb - i * kAtoms);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk)
-          mma_bf16(tmem, sdesc(sa + kk * 32), sdesc(sb + kk * 32), idesc,
-                   (i > 0 || kk > 0) ? 1u : 0u);
+        for (int a = 0; a < kAtoms; ++a) {
+          if (a < na) {
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk)
+              mma_bf16(tmem, sdesc(sa + a * A_ATOM + kk * 32), sdesc(sb + a * B_ATOM + kk * 32), idesc,
+                       (i > 0 || a > 0 || kk > 0) ? 1u : 0u);
+          }
+        }
         mma_commit(smem_u32(&bars[STAGES + s]));
       }
       if (ok) mma_commit(smem_u32(&bars[2 * STAGES]));
@@ -239,6 +259,19 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
               *reinterpret_cast<float4*>(T + lane * 68 + 32 * h2 + 4 * q) =
                   make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
           }
+          // residuals of all this warp's rows first (EPI_RESID)
+          float4 xlo[EPI == EPI_RESID ? NI : 1], xhi[EPI == EPI_RESID ? NI : 1];
+          if (EPI == EPI_RESID) {
+#pragma unroll
+            for (int ii = 0; ii < NI; ++ii) {
+              const int row = m0 + quarter * 32 + gr + 4 * (ibase + ii);
+              const float* xp = g.epi.x + (size_t)row * g.epi.ldx + n0 + c + gc;
+              const bool okr = row < g.M && n0 + c + gc < g.N;
+              xlo[ii] = okr ? *reinterpret_cast<const float4*>(xp) : make_float4(0.f, 0.f, 0.f, 0.f);
+              xhi[ii] = (okr && n0 + c + 32 + gc < g.N) ? *reinterpret_cast<const float4*>(xp + 32)
+                                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+          }
           __syncwarp();
 #pragma unroll
           for (int ii = 0; ii < NI; ++ii) {
@@ -256,6 +289,10 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
             if (ok) {
               if (EPI == EPI_QKV) {
                 epi_qkv<__nv_bfloat16>(g.epi, row, meta->pos[rl], meta->aux[rl], n0 + c, gc, lo, hi);
+              } else if (EPI == EPI_RESID) {
+                if (n0 + c + gc < g.N) sq = epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + gc, lo, xlo[ii]);
+                if (n0 + c + 32 + gc < g.N)
+                  sq += epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + 32 + gc, hi, xhi[ii]);
               } else {
                 sq = epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N) +
                      epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
@@ -311,6 +348,13 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
           off[u] = (uint32_t)((rr * (BN + 4) + gcol[u]) * 4);
           acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
+        float4 xo[EPI == EPI_RESID ? U : 1];
+        if (EPI == EPI_RESID) {
+#pragma unroll
+          for (int u = 0; u < U; ++u)
+            xo[u] = (ok[u] && n0 + gcol[u] < g.N) ? *reinterpret_cast<const float4*>(g.epi.x + (size_t)row[u] * g.epi.ldx + n0 + gcol[u])
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
         for (int sp = 0; sp < S; ++sp) {
 #pragma unroll
           for (int u = 0; u < U; ++u) {
@@ -324,7 +368,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
 #pragma unroll
           for (int u = 0; u < U; ++u) {
             if (EPI == EPI_BIAS_GELU && ok[u] && g.epi.ss_in) acc[u] = scale4(acc[u], meta->rinv[row[u] - m0]);
-            float sq = ok[u] ? epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N) : 0.f;
+            float sq = 0.f;
+            if (EPI == EPI_RESID) {
+              if (ok[u] && n0 + gcol[u] < g.N) sq = epi_resid4<__nv_bfloat16>(g.epi, row[u], n0 + gcol[u], acc[u], xo[u]);
+            } else {
+              sq = ok[u] ? epi_vec4<__nv_bfloat16, EPI>(g.epi, row[u], n0 + gcol[u], acc[u], g.N) : 0.f;
+            }
             if ((EPI == EPI_RESID || EPI == EPI_NOISE_OUT) && g.epi.ss_out) {
               // 16 consecutive lanes hold one row's 64-column slot
               sq += __shfl_xor_sync(0xffffffffu, sq, 1);
@@ -406,7 +455,7 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
     while (splits < 8 && tiles * splits * 2 <= num_sms && kb_total >= splits * 4) splits *= 2;
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
-  const size_t smem = (size_t)STAGES * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
+  const size_t smem = (size_t)STAGES * kAtoms * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
   static bool attr_set = false;
   if (!attr_set) {
     cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -495,8 +544,8 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
   // 64-wide tiles when they fit in one wave, else 128-wide (a second partial
   // wave costs more than the wider tile)
   const int tiles64 = ceil_div(g.N, 64) * ceil_div(g.M, kBM);
-  if (tiles64 <= num_sms) return launch_bn<64, 8>(g, d_err, num_sms, s);
-  return launch_bn<128, 6>(g, d_err, num_sms, s);
+  if (tiles64 <= num_sms) return launch_bn<64, 4>(g, d_err, num_sms, s);
+  return launch_bn<128, 3>(g, d_err, num_sms, s);
 }
 
 }  // namespace kf

@@ -237,6 +237,17 @@ __device__ __forceinline__ void st_ta4(__nv_bfloat16* p, float4 v) {
   *reinterpret_cast<uint2*>(p) = u;
 }
 
+// EPI_RESID with the residual x[row][col..+3] already loaded (xo): the
+// callers fetch every residual of a batch of outputs before any store, so
+// the loads are not serialised behind stores that might alias them
+template <typename TA>
+__device__ __forceinline__ float epi_resid4(const Epi& e, int row, int col, float4 v, float4 xo) {
+  v = make_float4(xo.x + v.x, xo.y + v.y, xo.z + v.z, xo.w + v.w);
+  *reinterpret_cast<float4*>(e.x + (size_t)row * e.ldx + col) = v;
+  if (e.xb_out) st_ta4(reinterpret_cast<TA*>(e.xb_out) + (size_t)row * e.ldx + col, v);
+  return v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+}
+
 template <typename TA, int EPI>
 __device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4 v, int N) {
   if (col >= N) return 0.f;

@@ -16,6 +16,7 @@ SHAPES = [
     (320, 3072, 768),    # first-step rows (P=1), MLP-up
     (256, 30720, 768),   # LM-head shape (vocab padded to 256)
     (1000, 200, 128),    # N not a multiple of the tile
+    (200, 640, 320),     # odd number of 64-wide K blocks: a short last pipeline stage
     (4096, 768, 3072),   # large M
 ]
 
