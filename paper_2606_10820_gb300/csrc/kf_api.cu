@@ -213,7 +213,8 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   // trips and V transpose cost more than FMA scores (measured), so those use
   // the CUDA-core kernel.
   const int rows = groups ? kMaxGroupRows : uniform_rows;
-  const bool tc_attn = c->fused && rows > 8;
+  const bool mma_attn = attention_mma_supported(c->bf16, c->hd, rows);
+  const bool tc_attn = !mma_attn && c->fused && rows > 8;
   int n_split, kps;
   attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
   auto norm_in = [&](Epi& e) {
@@ -255,7 +256,8 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     prof_begin(c, KF_KIND_ATTENTION);
-    if (tc_attn) launch_attention_tc(a, n_groups, s);
+    if (mma_attn) launch_attention_mma(a, n_groups, c->cfg.max_len, s);
+    else if (tc_attn) launch_attention_tc(a, n_groups, s);
     else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
     if (n_split > 1) {

@@ -22,6 +22,7 @@ constexpr int kErrBadToken = 1;
 constexpr int kErrBadPage = 2;
 constexpr int kErrTimeout = 4;
 constexpr int kErrBadRow = 8;
+constexpr int kErrInternal = 16;   // a launch invariant of the host plan did not hold
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 __host__ __device__ inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
@@ -368,6 +369,9 @@ struct AttnArgs {
 // max_keys: the most keys any row of the launch can see (max_len bound)
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
 void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
+// decode attention on warp-level MMA (bf16 cache, head_dim 64, <= 16 rows per group)
+bool attention_mma_supported(bool bf16, int hd, int rows);
+void launch_attention_mma(const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
 // tensor-core decode attention (bf16 cache, head_dim 64, <= 16 rows per group,
 // keys_per_split <= attention_tc_max_keys())
 void launch_attention_tc(const AttnArgs& a, int n_groups, cudaStream_t s);
