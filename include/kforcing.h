@@ -52,6 +52,9 @@ extern "C" {
 #define KF_FLAG_NO_GRAPH 1       /* launch kernels eagerly instead of replaying a CUDA graph */
 #define KF_FLAG_SIMT_GEMM 2      /* bf16 mode: use the SIMT GEMM, not tcgen05   */
 #define KF_FLAG_NO_PDL 4         /* launch without programmatic dependent launch */
+#define KF_FLAG_TC_ATTN 8        /* bf16, head_dim 64: attention of groups of more than 8
+                                    query rows on the tcgen05 kernel instead of the
+                                    warp-MMA kernel (kept for comparison)        */
 
 /*
  * Model and runtime configuration.  Table 4 gives the backbone (pre-norm

@@ -208,13 +208,13 @@ static void attn_plan(kf_ctx* c, int n_groups, int R, int max_keys, int* n_split
 static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, int uniform_rows) {
   const int d = c->d, H = c->H, F = c->F;
   cudaStream_t s = c->stream;
-  // Tensor-core attention on the fused bf16 path for groups of more than 8
-  // query rows (k = 8 steps, prefill); with 1..8 rows its per-tile MMA round
-  // trips and V transpose cost more than FMA scores (measured), so those use
-  // the CUDA-core kernel.
+  // Attention: the warp-MMA kernel for the bf16 cache with head_dim 64; the
+  // tcgen05 kernel for groups of more than 8 rows only on request
+  // (KF_FLAG_TC_ATTN, measured slower); the FP32-FMA kernel otherwise (fp32
+  // cache, head_dim 32).
   const int rows = groups ? kMaxGroupRows : uniform_rows;
-  const bool mma_attn = attention_mma_supported(c->bf16, c->hd, rows);
-  const bool tc_attn = !mma_attn && c->fused && rows > 8;
+  const bool tc_attn = c->fused && rows > 8 && (c->cfg.flags & KF_FLAG_TC_ATTN);
+  const bool mma_attn = !tc_attn && attention_mma_supported(c->bf16, c->hd, rows);
   int n_split, kps;
   attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
   auto norm_in = [&](Epi& e) {
@@ -256,8 +256,8 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     prof_begin(c, KF_KIND_ATTENTION);
-    if (mma_attn) launch_attention_mma(a, n_groups, c->cfg.max_len, s);
-    else if (tc_attn) launch_attention_tc(a, n_groups, s);
+    if (tc_attn) launch_attention_tc(a, n_groups, s);
+    else if (mma_attn) launch_attention_mma(a, n_groups, c->cfg.max_len, s);
     else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
     if (n_split > 1) {

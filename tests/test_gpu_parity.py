@@ -243,6 +243,19 @@ def test_lm1b_bf16_small_batch(kf, lm1b_weights):
     dec.close()
 
 
+@pytest.mark.parametrize("flags", [0, 8])   # 8 = KF_FLAG_TC_ATTN
+def test_lm1b_bf16_k8_both_attention_kernels(kf, lm1b_weights, flags):
+    """k = 8 (16 query rows per sequence) and ragged prefill groups on the
+    warp-MMA attention kernel and, with KF_FLAG_TC_ATTN, the tcgen05 one."""
+    cfg = LM1B
+    prompts = make_prompts([40, 23, 17], cfg.vocab)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [8, 8, 4, 8], max_k=8, flags=flags)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert worst <= LOGIT_TOL
+    assert bad == 0
+    dec.close()
+
+
 def test_lm1b_bf16_argmax(kf, lm1b_weights):
     cfg = LM1B.replace(map="argmax")
     prompts = make_prompts([32, 20], cfg.vocab)
