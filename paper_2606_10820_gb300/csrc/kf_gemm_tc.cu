@@ -36,8 +36,7 @@ namespace kf {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;                 // one 128-byte swizzle atom of bf16
-constexpr int kAtoms = 2;               // K atoms per pipeline stage (one wait and one
-                                        // commit per 8 MMAs)
+
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 
@@ -61,14 +60,20 @@ __device__ __forceinline__ void epi_bar() {
 }
 
 // ------------------------------------------------------------ the kernel
-template <int BN, int STAGES, int EPI>
+// MT: 128-row M tiles per CTA, each with its own TMEM accumulator (2 only for
+// the LM-head records, which need no per-row data); AT: 64-wide K atoms per
+// pipeline stage, so that one mbarrier wait and one commit cover 4 * MT * AT
+// MMAs
+template <int BN, int STAGES, int EPI, int MT, int AT>
 __global__ void __launch_bounds__(kThreads, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
           TcArgs g) {
   constexpr uint32_t A_ATOM = kBM * kBK * 2;            // one 128 x 64 A box
   constexpr uint32_t B_ATOM = BN * kBK * 2;             // one BN x 64 W box
-  constexpr uint32_t A_BYTES = kAtoms * A_ATOM;
-  constexpr uint32_t STAGE_BYTES = kAtoms * (A_ATOM + B_ATOM);   // [A atoms][W atoms]
+  constexpr uint32_t A_BYTES = AT * MT * A_ATOM;        // [atom][M tile] A boxes
+  constexpr uint32_t STAGE_BYTES = AT * (MT * A_ATOM + B_ATOM);   // [A boxes][W atoms]
+  constexpr int TMEM_COLS = MT * BN;
+  static_assert(MT == 1 || EPI == EPI_HEAD, "two M tiles per CTA only for the LM-head records");
   static_assert(kEpiWarps * 32 * 68 * 4 <= STAGES * STAGE_BYTES &&
                     kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
                 "epilogue blocks and split partials live in the idle pipeline stages");
@@ -84,12 +89,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_tile = blockIdx.x, m_tile = blockIdx.y, split = blockIdx.z;
-  const int n0 = n_tile * BN, m0 = m_tile * kBM;
+  const int n0 = n_tile * BN, m0 = m_tile * kBM * MT;
   const int kb_total = g.K / kBK;
   const int kb0 = split * g.kb_per_split;
   const int kb1 = min(kb_total, kb0 + g.kb_per_split);
   const int nkb = kb1 - kb0;                  // K atoms of this split
-  const int nst = (nkb + kAtoms - 1) / kAtoms; // pipeline stages (the last may be short)
+  const int nst = (nkb + AT - 1) / AT;        // pipeline stages (the last may be short)
   pdl_trigger();
 
   if (threadIdx.x == 0) {
@@ -105,7 +110,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(tmem_slot)),
-                 "r"(BN)
+                 "r"(TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -122,30 +127,32 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       const int pre = min(nst, STAGES);
       for (int i = 0; i < pre; ++i) {
         const uint32_t full = smem_u32(&bars[i]);
-        const int na = min(kAtoms, nkb - i * kAtoms);
-        mbar_expect_tx(full, na * (A_ATOM + B_ATOM));
+        const int na = min(AT, nkb - i * AT);
+        mbar_expect_tx(full, na * (MT * A_ATOM + B_ATOM));
         for (int a = 0; a < na; ++a)
           tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES + a * B_ATOM, &map_w, full,
-                      (kb0 + i * kAtoms + a) * kBK, n0);
+                      (kb0 + i * AT + a) * kBK, n0);
       }
       pdl_wait();
       for (int i = 0; i < pre; ++i) {
-        const int na = min(kAtoms, nkb - i * kAtoms);
+        const int na = min(AT, nkb - i * AT);
         for (int a = 0; a < na; ++a)
-          tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + a * A_ATOM, &map_a, smem_u32(&bars[i]),
-                      (kb0 + i * kAtoms + a) * kBK, m0);
+          for (int mh = 0; mh < MT; ++mh)
+            tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + (a * MT + mh) * A_ATOM, &map_a,
+                        smem_u32(&bars[i]), (kb0 + i * AT + a) * kBK, m0 + mh * kBM);
       }
       for (int i = pre; i < nst; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (i / STAGES) & 1;
         if (!mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, g.d_err)) break;
         const uint32_t full = smem_u32(&bars[s]);
-        const int na = min(kAtoms, nkb - i * kAtoms);
-        mbar_expect_tx(full, na * (A_ATOM + B_ATOM));
+        const int na = min(AT, nkb - i * AT);
+        mbar_expect_tx(full, na * (MT * A_ATOM + B_ATOM));
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
         for (int a = 0; a < na; ++a) {
-          const int kc = (kb0 + i * kAtoms + a) * kBK;
-          tma_load_2d(sa + a * A_ATOM, &map_a, full, kc, m0);
+          const int kc = (kb0 + i * AT + a) * kBK;
+          for (int mh = 0; mh < MT; ++mh)
+            tma_load_2d(sa + (a * MT + mh) * A_ATOM, &map_a, full, kc, m0 + mh * kBM);
           tma_load_2d(sa + A_BYTES + a * B_ATOM, &map_w, full, kc, n0);
         }
       }
@@ -161,14 +168,16 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
         const uint32_t sb = sa + A_BYTES;
-        const int na = min(kAtoms, nkb - i * kAtoms);
+        const int na = min(AT, nkb - i * AT);
 #pragma unroll
-        for (int a = 0; a < kAtoms; ++a) {
+        for (int a = 0; a < AT; ++a) {
           if (a < na) {
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-              mma_bf16(tmem, sdesc(sa + a * A_ATOM + kk * 32), sdesc(sb + a * B_ATOM + kk * 32), idesc,
-                       (i > 0 || a > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+              for (int mh = 0; mh < MT; ++mh)
+                mma_bf16(tmem + mh * BN, sdesc(sa + (a * MT + mh) * A_ATOM + kk * 32),
+                         sdesc(sb + a * B_ATOM + kk * 32), idesc, (i > 0 || a > 0 || kk > 0) ? 1u : 0u);
           }
         }
         mma_commit(smem_u32(&bars[STAGES + s]));
@@ -227,13 +236,16 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
                 make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
       } else if (EPI == EPI_HEAD) {
-        // row mode: a thread reduces its row's 32-id chunks (alternate
-        // halves of the tile's columns per warp of the quarter)
-        const int row = rbase + lane;
+        // row mode: a thread reduces its row's 32-id chunks; with two M
+        // tiles the warps of a quarter take one accumulator each, else
+        // alternate halves of the tile's columns
+        const int row = rbase + (MT == 2 ? ch * kBM : 0) + lane;
+        const int c0 = MT == 2 ? 0 : ch * (BN / 2), c1 = MT == 2 ? BN : (ch + 1) * (BN / 2);
+        const uint32_t acc_addr = lane_addr + (MT == 2 ? ch * BN : 0);
 #pragma unroll 1
-        for (int c = ch * (BN / 2); c < (ch + 1) * (BN / 2); c += 32) {
+        for (int c = c0; c < c1; c += 32) {
           float v[32];
-          tmem_ld32(lane_addr + c, v);
+          tmem_ld32(acc_addr + c, v);
           if (row < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, row, n0 + c, v, g.N);
         }
       } else {
@@ -395,7 +407,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (warp == 1)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS)
                  : "memory");
 }
 
@@ -442,9 +454,9 @@ bool tc_gemm_supported(const GemmDesc& g) {
   return get_encode();
 }
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, int MT = 1, int AT = 2>
 static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s) {
-  const int n_tiles = ceil_div(g.N, BN), m_tiles = ceil_div(g.M, kBM);
+  const int n_tiles = ceil_div(g.N, BN), m_tiles = ceil_div(g.M, kBM * MT);
   const int tiles = n_tiles * m_tiles;
   const int kb_total = g.K / kBK;
   // split K over a cluster of up to 8 CTAs when the tiles alone leave SMs
@@ -455,10 +467,10 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
     while (splits < 8 && tiles * splits * 2 <= num_sms && kb_total >= splits * 4) splits *= 2;
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
-  const size_t smem = (size_t)STAGES * kAtoms * (kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
+  const size_t smem = (size_t)STAGES * AT * (MT * kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
   static bool attr_set = false;
   if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI, MT, AT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     attr_set = true;
   }
@@ -477,7 +489,7 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
       q.attrs = &ca;
       q.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<BN, STAGES, EPI>, &q) == cudaSuccess && n > 0) {
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<BN, STAGES, EPI, MT, AT>, &q) == cudaSuccess && n > 0) {
         max_cluster = cs;
         break;
       }
@@ -516,7 +528,7 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
   }
   cfg.attrs = at;
   cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN, STAGES, EPI>, ma, mw, a) == cudaSuccess ? 0 : -1;
+  return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN, STAGES, EPI, MT, AT>, ma, mw, a) == cudaSuccess ? 0 : -1;
 }
 
 template <int BN, int STAGES>
@@ -526,7 +538,6 @@ static int launch_bn(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s)
     case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU>(g, d_err, num_sms, s);
     case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID>(g, d_err, num_sms, s);
     case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT>(g, d_err, num_sms, s);
-    case EPI_HEAD: return launch_epi<BN, STAGES, EPI_HEAD>(g, d_err, num_sms, s);
     case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS>(g, d_err, num_sms, s);
     case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32>(g, d_err, num_sms, s);
     case EPI_QKV: return launch_epi<BN, STAGES, EPI_QKV>(g, d_err, num_sms, s);
@@ -540,6 +551,12 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  // LM-head records: 256-wide tiles; above 128 rows both M tiles of a row
+  // pair in one CTA (each weight tile is streamed from HBM once per 256 rows)
+  if (g.epi.kind == EPI_HEAD) {
+    if (g.M > kBM) return launch_epi<256, 3, EPI_HEAD, 2, 1>(g, d_err, num_sms, s);
+    return launch_epi<256, 2, EPI_HEAD, 1, 2>(g, d_err, num_sms, s);
   }
   // 64-wide tiles when they fit in one wave, else 128-wide (a second partial
   // wave costs more than the wider tile)

@@ -207,9 +207,21 @@ __device__ __forceinline__ void epi_run32(const Epi& e, int row, int col0, const
         if (j < nv && l > m) { m = l; a = col0 + j; }
       }
       float s = 0.f;
+      if (sizeof(TA) == 2) {
+        // bf16 path: the hardware 2^x on log2(e)-scaled differences (relative
+        // error ~2^-22 per term)
+        const float k2 = 1.4426950408889634f;
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (j < nv) s += expf(v[j] * e.inv_tau - m);
+        for (int j = 0; j < 32; ++j) {
+          float t;
+          asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"((v[j] * e.inv_tau - m) * k2));
+          if (j < nv) s += t;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (j < nv) s += expf(v[j] * e.inv_tau - m);
+      }
       HeadRec r;
       r.m = m; r.s = s; r.a = a; r.pad = 0;
       e.rec[(size_t)row * e.nchunk + col0 / 32] = r;
