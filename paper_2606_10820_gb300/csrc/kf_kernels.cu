@@ -340,12 +340,29 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   const int per = ceil_div(nchunk, kSelThreads);
   const int c0 = min(nchunk, t * per), c1 = min(nchunk, c0 + per);
 
-  // 1) M and (for argmax) the lowest id attaining it
+  // 1) M and (for argmax) the lowest id attaining it; the thread's records
+  //    stay in registers for step 2 when they fit
+  constexpr int kKeep = 8;
+  const bool keep = c1 - c0 <= kKeep;
+  float km[kKeep], ks[kKeep];
   float m = -INFINITY;
   int am = 0x7fffffff;
-  for (int c = c0; c < c1; ++c) {
-    HeadRec r = rec[c];
-    if (r.m > m) { m = r.m; am = r.a; }
+#pragma unroll
+  for (int i = 0; i < kKeep; ++i) {
+    km[i] = -INFINITY;
+    ks[i] = 0.f;
+    if (keep && c0 + i < c1) {
+      const HeadRec r = rec[c0 + i];
+      km[i] = r.m;
+      ks[i] = r.s;
+      if (r.m > m) { m = r.m; am = r.a; }
+    }
+  }
+  if (!keep) {
+    for (int c = c0; c < c1; ++c) {
+      HeadRec r = rec[c];
+      if (r.m > m) { m = r.m; am = r.a; }
+    }
   }
   for (int o = 16; o > 0; o >>= 1) {
     float m2 = __shfl_xor_sync(0xffffffffu, m, o);
@@ -369,50 +386,73 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   }
   const float M = s_M;
 
-  // 2) per-thread partial sums, then an ordered scan over threads
+  // 2) per-thread partial sums (id order inside each range), then a
+  //    fixed-order block scan over the threads: lanes by shuffles, warps by
+  //    their totals.  The scan's last element is the total S, so T = z S
+  //    is crossed for every z < 1.
   float part = 0.f;
-  for (int c = c0; c < c1; ++c) {
-    HeadRec r = rec[c];
-    part += r.s * expf(r.m - M);
+  if (keep) {
+#pragma unroll
+    for (int i = 0; i < kKeep; ++i)
+      if (c0 + i < c1) part += ks[i] * expf(km[i] - M);
+  } else {
+    for (int c = c0; c < c1; ++c) {
+      HeadRec r = rec[c];
+      part += r.s * expf(r.m - M);
+    }
   }
-  s_part[t] = part;
+  float inc = part;
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  float lane_excl = __shfl_up_sync(0xffffffffu, inc, 1);
+  if (lane == 0) lane_excl = 0.f;
+  if (lane == 31) s_red[warp] = inc;
   __syncthreads();
+  __shared__ float s_wexcl[kSelThreads / 32 + 1];
   if (t == 0) {
-    float S = 0.f;
-    for (int i = 0; i < kSelThreads; ++i) S += s_part[i];
-    float T = noise[row] * S;
-    // first thread range whose running sum passes T
     float run = 0.f;
-    int th = -1;
-    for (int i = 0; i < kSelThreads; ++i) {
-      if (run + s_part[i] > T) { th = i; break; }
-      run += s_part[i];
+    for (int w = 0; w < kSelThreads / 32; ++w) {
+      s_wexcl[w] = run;
+      run += s_red[w];
     }
-    int cstar = -1;
-    float before = 0.f;
-    if (th >= 0) {
-      int a0 = min(nchunk, th * per), a1 = min(nchunk, a0 + per);
-      float acc = run;
-      for (int c = a0; c < a1; ++c) {
-        HeadRec r = rec[c];
-        float sc = r.s * expf(r.m - M);
-        // the range's own order can round differently from its partial sum:
-        // its last chunk takes the crossing then
-        if (acc + sc > T || c == a1 - 1) { cstar = c; before = acc; break; }
-        acc += sc;
-      }
-    }
-    int fallback = 0;
-    if (cstar < 0) {
-      // no crossing at all (z near 1): the last chunk with mass, last id in it
-      cstar = nchunk - 1;
-      while (cstar > 0 && !(rec[cstar].s * expf(rec[cstar].m - M) > 0.f)) --cstar;
-      fallback = 1;
+    s_wexcl[kSelThreads / 32] = run;     // S
+    s_T = noise[row] * run;
+    s_redi[2] = kSelThreads;             // first crossing thread (none yet)
+  }
+  __syncthreads();
+  const float T = s_T;
+  const float excl = s_wexcl[warp] + lane_excl, incl = s_wexcl[warp] + inc;
+  {
+    const unsigned cross = __ballot_sync(0xffffffffu, incl > T);
+    if (lane == 0 && cross) atomicMin(&s_redi[2], warp * 32 + __ffs(cross) - 1);
+  }
+  __syncthreads();
+  if (t == s_redi[2]) {
+    // the crossing range: walk its chunks in id order from its exclusive prefix
+    float acc = excl;
+    int cstar = c1 - 1;
+    float before = acc;
+    for (int c = c0; c < c1; ++c) {
+      HeadRec r = rec[c];
+      const float sc = r.s * expf(r.m - M);
+      // the range's own order can round differently from its partial sum:
+      // its last chunk takes the crossing then
+      if (acc + sc > T || c == c1 - 1) { cstar = c; before = acc; break; }
+      acc += sc;
     }
     s_chunk = cstar;
     s_before = before;
-    s_T = T;
-    s_redi[1] = fallback;
+    s_redi[1] = 0;
+  }
+  if (t == 0 && s_redi[2] >= kSelThreads) {
+    // no crossing at all (z near 1): the last chunk with mass, last id in it
+    int cstar = nchunk - 1;
+    while (cstar > 0 && !(rec[cstar].s * expf(rec[cstar].m - M) > 0.f)) --cstar;
+    s_chunk = cstar;
+    s_before = 0.f;
+    s_redi[1] = 1;
   }
   __syncthreads();
 
@@ -421,24 +461,34 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   __shared__ float s_logit[kChunk];
   const int cstar = s_chunk;
   {
+    // the warp's NQ ids side by side, so their weight loads are in flight together
     const TA* hr = head_in + (size_t)row * d;
     constexpr int VEC = 16 / sizeof(TA);
-    for (int q = 0; q < kChunk / (kSelThreads / 32); ++q) {
-      const int jj = warp * (kChunk / (kSelThreads / 32)) + q;
-      const int v = cstar * kChunk + jj;
-      float acc = 0.f;
-      if (v < V) {
-        const TA* wr = w_head + (size_t)v * d;
-        for (int c0 = lane * VEC; c0 < d; c0 += 32 * VEC) {
-          float hv[VEC], wv[VEC];
-          ld_vec(hr + c0, hv);
-          ld_vec(wr + c0, wv);
+    constexpr int NQ = kChunk / (kSelThreads / 32);
+    const int jj0 = warp * NQ;
+    float acc[NQ];
 #pragma unroll
-          for (int i = 0; i < VEC; ++i) acc = fmaf(hv[i], wv[i], acc);
+    for (int q = 0; q < NQ; ++q) acc[q] = 0.f;
+    for (int c0 = lane * VEC; c0 < d; c0 += 32 * VEC) {
+      float hv[VEC];
+      ld_vec(hr + c0, hv);
+#pragma unroll
+      for (int q = 0; q < NQ; ++q) {
+        const int v = cstar * kChunk + jj0 + q;
+        if (v < V) {
+          float wv[VEC];
+          ld_vec(w_head + (size_t)v * d + c0, wv);
+#pragma unroll
+          for (int i = 0; i < VEC; ++i) acc[q] = fmaf(hv[i], wv[i], acc[q]);
         }
       }
-      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-      if (lane == 0) s_logit[jj] = (v < V) ? acc * inv_tau : -INFINITY;
+    }
+#pragma unroll
+    for (int q = 0; q < NQ; ++q) {
+      float a = acc[q];
+      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+      const int v = cstar * kChunk + jj0 + q;
+      if (lane == 0) s_logit[jj0 + q] = (v < V) ? a * inv_tau : -INFINITY;
     }
   }
   __syncthreads();
