@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--gen", type=int, default=0, help="tokens per sequence (0: workload)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--no-ar", action="store_true", help="skip the k=1 AR leg")
+    p.add_argument("--sweep-only", default="",
+                   help="comma-separated workload names: run only these sweep configurations")
     p.add_argument("--sweep", action="store_true",
                    help="one line per configuration: OWT-shaped batch 1..256, OWT paged "
                         "batch 512, medium batch 256 (k vs the AR step)")
@@ -266,8 +268,10 @@ def run_sweep(args):
     kf.load_library()
     pk, peak_src = peaks()
     by_wl = {}
+    only = [x for x in args.sweep_only.split(",") if x]
     for name, B, ks in SWEEP:
-        by_wl.setdefault(name, []).append((B, ks))
+        if not only or name in only:
+            by_wl.setdefault(name, []).append((B, ks))
     for name, runs in by_wl.items():
         w = WORKLOADS[name]
         model = w.model

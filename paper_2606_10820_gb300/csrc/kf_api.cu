@@ -255,6 +255,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.row_seq = c->row_seq; a.row_pos = c->row_pos; a.groups = groups;
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
+    a.len = groups ? nullptr : c->d_len;   // decode: keys below it are stable during the step
     prof_begin(c, KF_KIND_ATTENTION);
     if (tc_attn) launch_attention_tc(a, n_groups, s);
     else if (mma_attn) launch_attention_mma(a, n_groups, c->cfg.max_len, s);

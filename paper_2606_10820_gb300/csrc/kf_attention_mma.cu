@@ -91,42 +91,56 @@ constexpr size_t smem_bytes(int nbuf) {
 
 }  // namespace
 
-// NBUF = 1: CTAs of at most one key tile; NBUF = 2: double-buffered tiles
+// NBUF = 1: CTAs of at most one key tile; NBUF = 2: double-buffered tiles.
+// Single-tile decode CTAs (a.len set, one group per sequence): the keys before the
+// sequence's committed length were written by earlier steps and the page
+// table by the host before the step, so the copies of those keys are issued
+// before waiting for the kernel that appends this step's keys; the new keys
+// and Q are loaded after the wait.
 template <int NBUF>
 __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnArgs a) {
   pdl_trigger();
-  pdl_wait();
   extern __shared__ __align__(128) uint8_t sm[];
   __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(sm);   // [16][64] swizzled
   __nv_bfloat16* Ks = Qs + kQRows * kHD;                      // [NBUF][128][64] swizzled
   __nv_bfloat16* Vs = Ks + NBUF * kTile * kHD;                // [NBUF][128][64] swizzled
 
   const int gi = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
-  int b, row0, nr;
-  if (a.groups) {
-    const int4 gg = a.groups[gi];
-    b = gg.x; row0 = gg.y; nr = gg.z;
-  } else {
+  // (single-tile CTAs only: with several tiles the double buffer hides the
+  // first tile's latency already)
+  const bool early = NBUF == 1 && a.len != nullptr && a.groups == nullptr;
+  int b, row0, nr, n_keys, stable;
+  if (early) {
     b = gi; row0 = gi * a.uniform_rows; nr = a.uniform_rows;
+    stable = a.len[b];                       // committed length: positions row_pos of the step
+    n_keys = stable + nr;
+  } else {
+    pdl_wait();
+    if (a.groups) {
+      const int4 gg = a.groups[gi];
+      b = gg.x; row0 = gg.y; nr = gg.z;
+    } else {
+      b = gi; row0 = gi * a.uniform_rows; nr = a.uniform_rows;
+    }
+    n_keys = a.row_pos[row0 + nr - 1] + 1;
+    stable = 0;
   }
-  const int n_keys = a.row_pos[row0 + nr - 1] + 1;
   const int k_begin = split * a.keys_per_split;
   const int k_end = min(n_keys, k_begin + a.keys_per_split);
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int g = lane >> 2, tq = lane & 3;     // MMA fragment row group / column pair
-  const int pos0 = g < nr ? a.row_pos[row0 + g] : -1;          // rows g and g + 8
-  const int pos1 = g + 8 < nr ? a.row_pos[row0 + g + 8] : -1;
 
   const __nv_bfloat16* kv = reinterpret_cast<const __nv_bfloat16*>(a.kv);
   const size_t head_page = (size_t)kPage * kHD;
   const size_t layer_base = (size_t)a.layer * a.n_pages * 2 * a.H * head_page;
   bool bad_page = false;
 
-  // cp.async of the K and V tile starting at key kt into buffer buf
-  // (kt is a multiple of the page size: thread t copies chunk t % 8 of keys
-  // kt + t / 8 + 16 q, i.e. one key of page kt / 16 + q for q = 0..7; the page
-  // ids are all fetched before the first copy is issued)
-  auto load_tile = [&](int kt, int buf) {
+  // cp.async of the keys [key_lo, key_hi) of the tile starting at kt into
+  // buffer buf (keys >= k_end are zero-filled).  kt is a multiple of the page
+  // size: thread t copies chunk t % 8 of keys kt + t / 8 + 16 q, i.e. one key
+  // of page kt / 16 + q for q = 0..7; the page ids are all fetched before the
+  // first copy is issued.
+  auto load_tile = [&](int kt, int buf, int key_lo, int key_hi) {
     __nv_bfloat16* kd = Ks + (size_t)buf * kTile * kHD;
     __nv_bfloat16* vd = Vs + (size_t)buf * kTile * kHD;
     constexpr int NQ = kTile * 8 / kThr;
@@ -135,13 +149,16 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
 #pragma unroll
     for (int q = 0; q < NQ; ++q) {
       const int pi = kt / kPage + q;
-      pg[q] = (kt + q * kPage < k_end && pi < a.max_pages) ? __ldg(a.page_table + b * a.max_pages + pi) : -1;
+      const int kq = kt + q * kPage;        // first key of the page
+      pg[q] = (kq < k_end && kq + kPage > key_lo && kq < key_hi && pi < a.max_pages)
+                  ? __ldg(a.page_table + b * a.max_pages + pi) : -1;
     }
 #pragma unroll
     for (int q = 0; q < NQ; ++q) {
       const int idx = t + q * kThr;
       const int j = idx >> 3, c = idx & 7;
       const int key = kt + j;
+      if (key < key_lo || key >= key_hi) continue;
       const __nv_bfloat16* src = kv;
       int nbytes = 0;
       if (key < k_end) {
@@ -165,7 +182,17 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
     if (t == 0) atomicOr(a.d_err, kErrInternal);
     n_tiles = 1;
   }
-  if (n_tiles > 0) load_tile(k_begin, 0);   // first tile in flight while Q loads
+  if (n_tiles > 0) {
+    // first tile: its stable keys now, the rest after the wait
+    const int split_key = early ? max(k_begin, min(stable, k_begin + kTile)) : k_begin;
+    if (split_key > k_begin) load_tile(k_begin, 0, k_begin, split_key);
+    if (early) pdl_wait();
+    load_tile(k_begin, 0, split_key, k_begin + kTile);
+  } else if (early) {
+    pdl_wait();
+  }
+  const int pos0 = g < nr ? a.row_pos[row0 + g] : -1;          // rows g and g + 8
+  const int pos1 = g + 8 < nr ? a.row_pos[row0 + g + 8] : -1;
   {
     // Q rows scaled by log2(e) / sqrt(hd) (scores in base-2 units for ex2)
     // as bf16; rows >= nr are zero
@@ -198,7 +225,7 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
     const int kt = k_begin + it * kTile;
     const int buf = (NBUF == 2) ? (it & 1) : 0;
     if (NBUF == 2 && it + 1 < n_tiles) {
-      load_tile(kt + kTile, buf ^ 1);
+      load_tile(kt + kTile, buf ^ 1, kt + kTile, kt + 2 * kTile);
       cp_wait<1>();
     } else {
       cp_wait<0>();

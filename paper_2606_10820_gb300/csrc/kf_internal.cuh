@@ -377,6 +377,8 @@ struct AttnArgs {
   int n_split;
   int keys_per_split;      // multiple of 64
   int* d_err;
+  const int32_t* len = nullptr;  // decode: committed length per sequence (keys below it are
+                                 // not written during the step), or NULL
 };
 // max_keys: the most keys any row of the launch can see (max_len bound)
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
