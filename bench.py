@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--gen", type=int, default=0, help="tokens per sequence (0: workload)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--no-ar", action="store_true", help="skip the k=1 AR leg")
+    p.add_argument("--serving", action="store_true",
+                   help="the G* teacher call and continuous batching (LM1B, batch 64)")
     p.add_argument("--sweep-only", default="",
                    help="comma-separated workload names: run only these sweep configurations")
     p.add_argument("--sweep", action="store_true",
@@ -354,10 +356,115 @@ def run_sweep(args):
     return 0
 
 
+def run_serving(args):
+    """The serving entry points on the LM1B-shaped model, batch 64 (rank 0, N = 1):
+    the G* teacher call (k AR steps in one graph) against k separate AR calls,
+    and continuous batching: every finished sequence is replaced by a new
+    request at the step boundary (kf_admit), pages recycled; throughput
+    counts the requests' generated tokens and includes the admissions."""
+    import torch
+    from paper_2606_10820_gb300 import build as kbuild
+    from paper_2606_10820_gb300 import kforcing as kf
+    from synth import WORKLOADS, make_requests, make_weights, workload_prompts
+    kbuild.build()
+    kf.load_library()
+    w = WORKLOADS["lm1b"]
+    model, B, k, gen = w.model, w.batch, 4, w.gen_len
+    weights = make_weights(model)
+    stream = torch.cuda.Stream()
+    dec = kf.Decoder(model, weights, max_batch=B, max_k=k, stream=stream.cuda_stream)
+    dec.prefill(workload_prompts(w, B))
+    calls = gen // k
+    z = torch.rand((calls, B, k), device="cuda")
+    zc = z.permute(0, 2, 1).contiguous()            # [calls][k][B]: AR call j of block i
+    o = torch.zeros((calls, B, k), dtype=torch.int32, device="cuda")
+    o1 = torch.zeros((calls, k, B), dtype=torch.int32, device="cuda")
+
+    def teacher():
+        dec.rewind()
+        for i in range(calls):
+            kf.kf_teacher_step(dec.ctx, B, k, z[i], o[i])
+
+    def ar_calls():
+        dec.rewind()
+        for i in range(calls):
+            for j in range(k):
+                kf.kf_decode_step(dec.ctx, B, 0, zc[i, j], o1[i, j])
+
+    def timed(fn):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / args.steps
+
+    ms_t, ms_a = timed(teacher), timed(ar_calls)
+    toks = B * calls * k
+    print(json.dumps({"metric": "G* teacher tokens/s (k AR steps per call)", "unit": "tokens/s",
+                      "value": toks / (ms_t / 1e3), "ar_calls_value": toks / (ms_a / 1e3),
+                      "ms_per_generation": ms_t, "ar_calls_ms_per_generation": ms_a,
+                      "config": {"workload": "lm1b", "batch": B, "k": k, "gen_tokens_per_seq": gen},
+                      "data": "synthetic", "dtype": "bf16"}))
+
+    # continuous batching: requests of prompt 32 and 32..96 generated tokens
+    n_req = 4 * B
+    reqs = make_requests(n_req, w.prompt_len, 32, gen, k, model.vocab)
+    zr = torch.rand((64, B, k), device="cuda")
+    orr = torch.zeros((B, k), dtype=torch.int32, device="cuda")
+    for rep in range(2):                             # the second pass is timed
+        dec.prefill([r[0] for r in reqs[:B]])
+        left = [r[1] for r in reqs[:B]]
+        nxt, done, produced, steps, adm_s, n_calls = B, 0, 0, 0, 0.0, 0
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        while done < n_req:
+            kf.kf_decode_step(dec.ctx, B, k, zr[steps % 64], orr)
+            steps += 1
+            slots, prompts = [], []
+            for b in range(B):
+                if left[b] > 0:
+                    produced += min(k, left[b])
+                    left[b] -= k
+                    if left[b] <= 0:
+                        done += 1
+                        slots.append(b)
+                        if nxt < n_req:
+                            prompts.append(reqs[nxt][0])
+                            left[b] = reqs[nxt][1]
+                            nxt += 1
+                        else:
+                            # no request left: an idle slot restarts a short prompt
+                            # (not counted) so its length stays within max_len
+                            prompts.append(reqs[0][0][:k])
+            if slots:
+                ta = time.perf_counter()
+                dec.admit(slots, prompts)          # all of this step's finished slots at once
+                adm_s += time.perf_counter() - ta
+                n_calls += 1
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    print(json.dumps({"metric": "continuous batching: generated tokens/s with admissions",
+                      "unit": "tokens/s", "value": produced / wall, "requests": n_req,
+                      "decode_steps": steps, "admissions": n_req, "admit_calls": n_calls,
+                      "admit_ms_per_call": 1e3 * adm_s / max(1, n_calls),
+                      "config": {"workload": "lm1b", "slots": B, "k": k, "prompt_len": w.prompt_len,
+                                 "gen_len": [32, gen]},
+                      "data": "synthetic", "dtype": "bf16", "timing": "host wall clock (admissions synchronise)"}))
+    dec.close()
+    return 0
+
+
 def main():
     args = parse()
     if args.sweep:
         return run_sweep(args)
+    if args.serving:
+        return run_serving(args)
     if args.impl == "reference":
         return run_reference(args)
     import torch

@@ -148,6 +148,41 @@ int kf_decode_step(kf_ctx* ctx, int32_t B, int32_t k, const float* noise,
                    int32_t* out_tokens);
 
 /*
+ * The k-pass teacher G* (App. B, Eq. sequential-icdf): k AR steps (Eq. 1
+ * with one token each) in one call, the j-th mapping the AR distribution
+ * conditioned on the cache, the pending tokens and the j-1 tokens drawn
+ * before it with noise[b][j].  The first sub-step feeds the P pending
+ * tokens, the later ones the token just drawn.  This is the target map the
+ * push-forward step learns; a caller uses it to produce teacher samples or to
+ * compare the joint step with the AR chain on the same noise.
+ * noise:      [B][k] fp32 in [0,1), host or device.
+ * out_tokens: [B][k] int32, host or device, caller-owned.
+ * Afterwards each cache holds P + k - 1 more tokens and the last drawn token
+ * is the one pending token.  1 <= k <= max_k.  Tokens equal those of k
+ * kf_decode_step calls with k = 0 on the same noise columns.  Errors as
+ * kf_decode_step.
+ */
+int kf_teacher_step(kf_ctx* ctx, int32_t B, int32_t k, const float* noise,
+                    int32_t* out_tokens);
+
+/*
+ * Continuous batching (App. C.1, KV-cached inference): at a step boundary,
+ * replace the n sequences slots[0..n) (distinct, 0 <= slot < B) by new
+ * prompts.  tokens is the concatenation of the n prompts (host or device),
+ * lens[i] their lengths (host).  The replaced sequences' KV pages return to
+ * the pool (recycled by later allocations); each new prompt is admitted with
+ * its first len - P tokens cached (one chunked prefill pass over all of
+ * them) and its last P tokens pending, P being the batch's current pending
+ * count, so every sequence keeps the same stride and the next kf_decode_step
+ * serves it like the others.  Synchronises.  lens[i] >= max(1, P).  After
+ * an admission kf_rewind is refused (KF_E_STATE) until the next kf_prefill.
+ * Errors: KF_E_ARG, KF_E_STATE, KF_E_CAPACITY (pool exhausted, or a prompt
+ * longer than max_len - 1), KF_E_CUDA, KF_E_DEVICE.
+ */
+int kf_admit(kf_ctx* ctx, int32_t n, const int32_t* slots, const int32_t* tokens,
+             const int32_t* lens);
+
+/*
  * Parity aid: recompute the last decode step's head logits (logits / tau,
  * fp32) for its B * max(k,1) mapped rows into out [B][max(k,1)][V] (host or
  * device).  The logits come from the same normalised rows and head weights

@@ -129,6 +129,22 @@ class OracleDecoder:
             self.seqs.append({"committed": p[:-1], "pending": p[-1:],
                               "cache": cache})
 
+    def admit(self, b: int, prompt, n_pending: int):
+        """Replace sequence b by a new prompt at a step boundary, its last
+        n_pending tokens pending (continuous batching, App. C.1: every
+        sequence of the batch keeps the same stride).  With n_pending = 1
+        this is prefill of that prompt alone."""
+        p = [int(t) for t in prompt]
+        assert 1 <= n_pending <= len(p)
+        n = len(p) - n_pending
+        cache = self.m.empty_cache()
+        if n > 0:
+            pos = np.arange(n)
+            h = self.m.token_rows(p[:n], pos)
+            _, new = self.m.forward(h, pos, cache)
+            cache = [(k, v) for (k, v) in new]
+        self.seqs[b] = {"committed": p[:n], "pending": p[n:], "cache": cache}
+
     def cached_len(self, b: int) -> int:
         return len(self.seqs[b]["committed"])
 

@@ -63,6 +63,7 @@ struct kf_ctx {
   std::vector<int> n_alloc;
   // sequence state
   bool have_batch = false, have_step = false;
+  bool admitted = false;        // kf_admit since the last kf_prefill (no rewind snapshot)
   int B = 0, P = 0, last_nh = 0;
   std::vector<int> h_len, h_len0;
   int32_t *d_len = nullptr, *d_len0 = nullptr, *d_pending = nullptr, *d_pending0 = nullptr;
@@ -78,6 +79,7 @@ struct kf_ctx {
   HeadRec* rec = nullptr;
   int nchunk = 0;
   int32_t* tokens = nullptr;
+  int32_t* t_out = nullptr;     // kf_teacher_step: [B][k] tokens of the k AR sub-steps
   float* noise = nullptr;
   int32_t *row_seq = nullptr, *row_pos = nullptr, *noise_map = nullptr, *head_map = nullptr;
   int32_t* row_tok = nullptr;
@@ -288,7 +290,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
 
 // One decode step on the device: no host data dependence, so it can be
 // captured once per (B, P, k) and replayed.
-static void enqueue_step(kf_ctx* c, int B, int P, int k) {
+static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   cudaStream_t s = c->stream;
   PdlScope pdl(!c->prof && !(c->cfg.flags & KF_FLAG_NO_PDL));
   const int d = c->d;
@@ -301,7 +303,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k) {
                        c->row_pos, c->V, d, c->x, c->fused ? c->xn : nullptr,
                        c->fused ? c->ss : nullptr, c->d_err, s);
   if (k > 0)
-    launch_noise_feat(c->bf16, B * k, c->noise, c->noise_freq, c->cfg.tau, c->cfg.noise_scale, d,
+    launch_noise_feat(c->bf16, B * k, noise, c->noise_freq, c->cfg.tau, c->cfg.noise_scale, d,
                       c->nfeat, s);
   prof_end(c);
   if (k > 0) {
@@ -325,7 +327,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k) {
   gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, d, c->head_in, d, c->w_head, d, eh);
   prof_begin(c, KF_KIND_HEAD_SELECT);
   launch_head_select(c->bf16, nh, c->rec, c->nchunk, c->head_in, d, c->w_head, c->V,
-                     1.0f / c->cfg.tau, c->cfg.map_kind, c->noise, c->tokens, s);
+                     1.0f / c->cfg.tau, c->cfg.map_kind, noise, c->tokens, s);
   prof_end(c);
   prof_begin(c, KF_KIND_COMMIT);
   launch_commit(B, P, k, c->tokens, c->d_pending, c->pend_stride, c->d_len, s);
@@ -547,6 +549,7 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
       (r = wbuf(&c->head_in, (size_t)c->NR_cap * d)) ||
       (r = dalloc(c, &c->rec, (size_t)c->NR_cap * c->nchunk * sizeof(HeadRec))) ||
       (r = dalloc(c, &c->tokens, (size_t)c->NR_cap * 4)) ||
+      (r = dalloc(c, &c->t_out, (size_t)c->NR_cap * 4)) ||
       (r = dalloc(c, &c->noise, (size_t)c->NR_cap * 4)) ||
       (r = dalloc(c, &c->row_seq, (size_t)R * 4)) || (r = dalloc(c, &c->row_pos, (size_t)R * 4)) ||
       (r = dalloc(c, &c->row_tok, (size_t)R * 4)) ||
@@ -567,6 +570,55 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
   if (e != cudaSuccess) { cuda_fail(c, e, "init"); return bail(KF_E_CUDA); }
   *out = c;
   return KF_OK;
+}
+
+// Prefill: the KV of each listed slot's first n tokens (positions 0..n-1),
+// in row chunks of up to prefill_rows, attention groups of <= 16 rows per
+// sequence.  The slots' pages must be allocated and uploaded.
+struct PrefillSeq {
+  int slot;
+  const int32_t* tok;
+  int n;
+};
+static int prefill_rows(kf_ctx* c, const std::vector<PrefillSeq>& seqs) {
+  std::vector<int32_t> r_tok, r_seq, r_pos;
+  std::vector<int4> grp;
+  auto flush = [&]() -> int {
+    int R = (int)r_tok.size();
+    if (R == 0) return KF_OK;
+    KF_CUDA(cudaMemcpyAsync(c->row_tok, r_tok.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
+    KF_CUDA(cudaMemcpyAsync(c->row_seq, r_seq.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
+    KF_CUDA(cudaMemcpyAsync(c->row_pos, r_pos.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
+    KF_CUDA(cudaMemcpyAsync(c->groups, grp.data(), grp.size() * sizeof(int4), cudaMemcpyHostToDevice,
+                            c->stream));
+    {
+      PdlScope pdl(!(c->cfg.flags & KF_FLAG_NO_PDL));
+      launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
+                          c->x, c->fused ? c->xn : nullptr, c->fused ? c->ss : nullptr, c->d_err,
+                          c->stream);
+      enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
+    }
+    KF_CUDA(cudaGetLastError());
+    // the host vectors are reused: wait until the copies have consumed them
+    KF_CUDA(cudaStreamSynchronize(c->stream));
+    r_tok.clear(); r_seq.clear(); r_pos.clear(); grp.clear();
+    return KF_OK;
+  };
+  for (const PrefillSeq& q : seqs) {
+    int p = 0;
+    while (p < q.n) {
+      if ((int)r_tok.size() == c->prefill_rows) KF_TRY(flush());
+      int take = std::min({q.n - p, kMaxGroupRows, c->prefill_rows - (int)r_tok.size()});
+      grp.push_back(make_int4(q.slot, (int)r_tok.size(), take, 0));
+      for (int i = 0; i < take; ++i) {
+        r_tok.push_back(q.tok[p + i]);
+        r_seq.push_back(q.slot);
+        r_pos.push_back(p + i);
+      }
+      p += take;
+    }
+  }
+  return flush();
 }
 
 int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens) {
@@ -600,54 +652,22 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
   KF_CUDA(cudaMemcpyAsync(c->d_page_table, c->h_page_table,
                           (size_t)c->cfg.max_batch * c->max_pages * 4, cudaMemcpyHostToDevice,
                           c->stream));
-  // rows: every prompt token but the last, chunked; attention groups of <= 16
-  std::vector<int32_t> r_tok, r_seq, r_pos;
-  std::vector<int4> grp;
-  auto flush = [&]() -> int {
-    int R = (int)r_tok.size();
-    if (R == 0) return KF_OK;
-    KF_CUDA(cudaMemcpyAsync(c->row_tok, r_tok.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
-    KF_CUDA(cudaMemcpyAsync(c->row_seq, r_seq.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
-    KF_CUDA(cudaMemcpyAsync(c->row_pos, r_pos.data(), R * 4, cudaMemcpyHostToDevice, c->stream));
-    KF_CUDA(cudaMemcpyAsync(c->groups, grp.data(), grp.size() * sizeof(int4), cudaMemcpyHostToDevice,
-                            c->stream));
-    {
-      PdlScope pdl(!(c->cfg.flags & KF_FLAG_NO_PDL));
-      launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
-                          c->x, c->fused ? c->xn : nullptr, c->fused ? c->ss : nullptr, c->d_err,
-                          c->stream);
-      enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
+  // rows: every prompt token but the last
+  std::vector<PrefillSeq> seqs;
+  {
+    size_t o = 0;
+    for (int b = 0; b < B; ++b) {
+      seqs.push_back({b, tok.data() + o, ln[b] - 1});
+      o += ln[b];
     }
-    KF_CUDA(cudaGetLastError());
-    // the host vectors are reused: wait until the copies have consumed them
-    KF_CUDA(cudaStreamSynchronize(c->stream));
-    r_tok.clear(); r_seq.clear(); r_pos.clear(); grp.clear();
-    return KF_OK;
-  };
-  size_t off = 0;
-  for (int b = 0; b < B; ++b) {
-    int n = ln[b] - 1;
-    int p = 0;
-    while (p < n) {
-      if ((int)r_tok.size() == c->prefill_rows) KF_TRY(flush());
-      int take = std::min({n - p, kMaxGroupRows, c->prefill_rows - (int)r_tok.size()});
-      grp.push_back(make_int4(b, (int)r_tok.size(), take, 0));
-      for (int i = 0; i < take; ++i) {
-        r_tok.push_back(tok[off + p + i]);
-        r_seq.push_back(b);
-        r_pos.push_back(p + i);
-      }
-      p += take;
-    }
-    off += ln[b];
   }
-  KF_TRY(flush());
+  KF_TRY(prefill_rows(c, seqs));
   // state: cached = N - 1, one pending token (the prompt's last)
   c->B = B;
   c->P = 1;
   c->h_len.assign(B, 0);
   std::vector<int32_t> pend((size_t)B * c->pend_stride, 0);
-  off = 0;
+  size_t off = 0;
   for (int b = 0; b < B; ++b) {
     c->h_len[b] = ln[b] - 1;
     pend[(size_t)b * c->pend_stride] = tok[off + ln[b] - 1];
@@ -664,6 +684,140 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
   KF_CUDA(cudaMemcpy(&err, c->d_err, 4, cudaMemcpyDeviceToHost));
   if (err) return fail(c, KF_E_DEVICE, "device error flag " + std::to_string(err) + " in prefill");
   c->have_batch = true;
+  c->admitted = false;
+  return KF_OK;
+}
+
+int kf_admit(kf_ctx* c, int32_t n, const int32_t* slots, const int32_t* tokens, const int32_t* lens) {
+  if (!c) return fail(nullptr, KF_E_ARG, "ctx is NULL");
+  if (!c->have_batch) return fail(c, KF_E_STATE, "admit before prefill");
+  if (n < 1 || n > c->B) return fail(c, KF_E_ARG, "n out of range 1..B");
+  if (!slots || !tokens || !lens) return fail(c, KF_E_ARG, "slots, tokens or lens is NULL");
+  const int P = c->P;
+  std::vector<int> sl(n), ln(n);
+  std::vector<char> seen(c->B, 0);
+  size_t total = 0;
+  for (int i = 0; i < n; ++i) {
+    sl[i] = slots[i];
+    ln[i] = lens[i];
+    if (sl[i] < 0 || sl[i] >= c->B) return fail(c, KF_E_ARG, "slot out of range 0..B-1");
+    if (seen[sl[i]]) return fail(c, KF_E_ARG, "slot listed twice");
+    seen[sl[i]] = 1;
+    if (ln[i] < 1 || ln[i] < P) return fail(c, KF_E_ARG, "prompt shorter than the batch's pending count");
+    if (ln[i] + 1 > c->cfg.max_len) return fail(c, KF_E_CAPACITY, "prompt longer than max_len - 1");
+    total += ln[i];
+  }
+  std::vector<int32_t> tok(total);
+  if (is_device_ptr(tokens)) {
+    KF_CUDA(cudaMemcpy(tok.data(), tokens, total * 4, cudaMemcpyDeviceToHost));
+  } else {
+    memcpy(tok.data(), tokens, total * 4);
+  }
+  for (size_t i = 0; i < total; ++i)
+    if (tok[i] < 0 || tok[i] >= c->V) return fail(c, KF_E_ARG, "token id out of range");
+  // steps in flight still read these slots' pages and the page-table mirror
+  KF_CUDA(cudaStreamSynchronize(c->stream));
+  // evict: the slots' pages return to the pool
+  for (int i = 0; i < n; ++i) {
+    const size_t row = (size_t)sl[i] * c->max_pages;
+    for (int j = 0; j < c->n_alloc[sl[i]]; ++j) {
+      c->free_pages.push_back(c->h_page_table[row + j]);
+      c->h_page_table[row + j] = -1;
+    }
+    c->n_alloc[sl[i]] = 0;
+  }
+  // insert: the first len - P tokens cached, the last P pending (the batch's
+  // pending count stays uniform)
+  std::vector<PrefillSeq> seqs;
+  std::vector<int32_t> pend((size_t)n * P), nl(n);
+  size_t off = 0;
+  for (int i = 0; i < n; ++i) {
+    const int m = ln[i] - P;
+    bool dirty = true;
+    if (m > 0) KF_TRY(ensure_pages(c, sl[i], m - 1, &dirty));
+    KF_TRY(upload_page_row(c, sl[i]));
+    if (m > 0) seqs.push_back({sl[i], tok.data() + off, m});
+    for (int j = 0; j < P; ++j) pend[(size_t)i * P + j] = tok[off + m + j];
+    nl[i] = m;
+    off += ln[i];
+  }
+  KF_TRY(prefill_rows(c, seqs));
+  for (int i = 0; i < n; ++i) {
+    KF_CUDA(cudaMemcpyAsync(c->d_pending + (size_t)sl[i] * c->pend_stride, pend.data() + (size_t)i * P,
+                            (size_t)P * 4, cudaMemcpyHostToDevice, c->stream));
+    KF_CUDA(cudaMemcpyAsync(c->d_len + sl[i], nl.data() + i, 4, cudaMemcpyHostToDevice, c->stream));
+    c->h_len[sl[i]] = nl[i];
+  }
+  KF_CUDA(cudaStreamSynchronize(c->stream));
+  int err = 0;
+  KF_CUDA(cudaMemcpy(&err, c->d_err, 4, cudaMemcpyDeviceToHost));
+  if (err) return fail(c, KF_E_DEVICE, "device error flag " + std::to_string(err) + " in admit");
+  c->admitted = true;
+  c->have_step = false;
+  return KF_OK;
+}
+
+int kf_teacher_step(kf_ctx* c, int32_t B, int32_t k, const float* noise, int32_t* out_tokens) {
+  if (!c) return fail(nullptr, KF_E_ARG, "ctx is NULL");
+  if (!c->have_batch) return fail(c, KF_E_STATE, "decode before prefill");
+  if (B != c->B) return fail(c, KF_E_ARG, "B differs from the prefilled batch");
+  if (k < 1 || k > c->max_k) return fail(c, KF_E_ARG, "k out of range 1..max_k");
+  if (!noise || !out_tokens) return fail(c, KF_E_ARG, "noise or out_tokens is NULL");
+  const int P = c->P;
+  for (int b = 0; b < B; ++b)
+    if (c->h_len[b] + P + k > c->cfg.max_len) return fail(c, KF_E_CAPACITY, "step would pass max_len");
+  for (int b = 0; b < B; ++b) {
+    bool dirty = false;
+    KF_TRY(ensure_pages(c, b, c->h_len[b] + P + k - 1, &dirty));
+    if (dirty) KF_TRY(upload_page_row(c, b));
+  }
+  // noise [B][k] -> [k][B]: sub-step j reads a contiguous column
+  for (int j = 0; j < k; ++j)
+    KF_CUDA(cudaMemcpy2DAsync(c->noise + (size_t)j * B, 4, noise + j, (size_t)k * 4, 4, B, cudaMemcpyDefault,
+                              c->stream));
+  // k AR sub-steps (Eq. 1 with k = 1, sequentially: the G* teacher of the
+  // k-token joint), each token copied into column j of t_out
+  auto enqueue = [&]() {
+    for (int j = 0; j < k; ++j) {
+      enqueue_step(c, B, j == 0 ? P : 1, 0, c->noise + (size_t)j * B);
+      cudaMemcpy2DAsync(c->t_out + j, (size_t)k * 4, c->tokens, 4, 4, B, cudaMemcpyDeviceToDevice, c->stream);
+    }
+  };
+  if (!(c->cfg.flags & KF_FLAG_NO_GRAPH)) {
+    auto key = std::make_tuple((int)B, P, -(int)k);
+    auto it = c->graphs.find(key);
+    cudaGraphExec_t exec = nullptr;
+    if (it == c->graphs.end()) {
+      cudaGraph_t g = nullptr;
+      KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
+      enqueue();
+      cudaError_t e1 = cudaGetLastError();
+      cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
+      if (e1 != cudaSuccess) return cuda_fail(c, e1, "capture launch");
+      if (e2 != cudaSuccess) return cuda_fail(c, e2, "cudaStreamEndCapture");
+      cudaError_t e3 = cudaGraphInstantiate(&exec, g, 0);
+      cudaGraphDestroy(g);
+      if (e3 != cudaSuccess) return cuda_fail(c, e3, "cudaGraphInstantiate");
+      c->graphs[key] = exec;
+    } else {
+      exec = it->second;
+    }
+    KF_CUDA(cudaGraphLaunch(exec, c->stream));
+  } else {
+    enqueue();
+    KF_CUDA(cudaGetLastError());
+  }
+  KF_CUDA(cudaMemcpyAsync(out_tokens, c->t_out, (size_t)B * k * 4, cudaMemcpyDefault, c->stream));
+  for (int b = 0; b < B; ++b) c->h_len[b] += P + k - 1;
+  c->P = 1;
+  c->last_nh = B;
+  c->have_step = true;
+  if (!is_device_ptr(out_tokens)) {
+    KF_CUDA(cudaStreamSynchronize(c->stream));
+    int err = 0;
+    KF_CUDA(cudaMemcpy(&err, c->d_err, 4, cudaMemcpyDeviceToHost));
+    if (err) return fail(c, KF_E_DEVICE, "device error flag " + std::to_string(err));
+  }
   return KF_OK;
 }
 
@@ -692,7 +846,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
     if (it == c->graphs.end()) {
       cudaGraph_t g = nullptr;
       KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
-      enqueue_step(c, B, P, k);
+      enqueue_step(c, B, P, k, c->noise);
       cudaError_t e1 = cudaGetLastError();
       cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
       if (e1 != cudaSuccess) return cuda_fail(c, e1, "capture launch");
@@ -715,7 +869,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
         for (auto& ev : c->ev) KF_CUDA(cudaEventCreate(&ev));
       }
     }
-    enqueue_step(c, B, P, k);
+    enqueue_step(c, B, P, k, c->noise);
     c->prof = false;
     KF_CUDA(cudaGetLastError());
   }
@@ -782,6 +936,7 @@ int kf_debug_logits(kf_ctx* c, float* out) {
 int kf_rewind(kf_ctx* c) {
   if (!c) return fail(nullptr, KF_E_ARG, "ctx is NULL");
   if (!c->have_batch) return fail(c, KF_E_STATE, "rewind before prefill");
+  if (c->admitted) return fail(c, KF_E_STATE, "rewind after kf_admit (no snapshot of admitted slots)");
   KF_CUDA(cudaMemcpyAsync(c->d_len, c->d_len0, c->B * 4, cudaMemcpyDeviceToDevice, c->stream));
   KF_CUDA(cudaMemcpyAsync(c->d_pending, c->d_pending0, (size_t)c->B * c->pend_stride * 4,
                           cudaMemcpyDeviceToDevice, c->stream));

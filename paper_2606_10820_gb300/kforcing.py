@@ -28,9 +28,9 @@ KIND_NAMES = ["rowmap", "embed", "noise_gemm", "rmsnorm", "gemm_qkv", "rope_kv",
               "head_select", "commit"]
 KF_KIND_COUNT = len(KIND_NAMES)
 
-EXPORTED = ["kf_init", "kf_prefill", "kf_decode_step", "kf_debug_logits", "kf_rewind",
-            "kf_get_lengths", "kf_set_stream", "kf_sync", "kf_profile_step", "kf_free",
-            "kf_last_error"]
+EXPORTED = ["kf_init", "kf_prefill", "kf_decode_step", "kf_teacher_step", "kf_admit",
+            "kf_debug_logits", "kf_rewind", "kf_get_lengths", "kf_set_stream", "kf_sync",
+            "kf_profile_step", "kf_free", "kf_last_error"]
 
 
 class KfError(RuntimeError):
@@ -72,6 +72,8 @@ def load_library(path: str = LIB_PATH):
                             ctypes.POINTER(P)]
     lib.kf_prefill.argtypes = [P, I32, VP, VP]
     lib.kf_decode_step.argtypes = [P, I32, I32, VP, VP]
+    lib.kf_teacher_step.argtypes = [P, I32, I32, VP, VP]
+    lib.kf_admit.argtypes = [P, I32, VP, VP, VP]
     lib.kf_debug_logits.argtypes = [P, VP]
     lib.kf_rewind.argtypes = [P]
     lib.kf_get_lengths.argtypes = [P, VP]
@@ -158,6 +160,14 @@ def kf_decode_step(ctx, B: int, k: int, noise, out_tokens):
     _check(load_library().kf_decode_step(ctx, B, k, _ptr(noise), _ptr(out_tokens)), ctx)
 
 
+def kf_teacher_step(ctx, B: int, k: int, noise, out_tokens):
+    _check(load_library().kf_teacher_step(ctx, B, k, _ptr(noise), _ptr(out_tokens)), ctx)
+
+
+def kf_admit(ctx, n: int, slots, tokens, lens):
+    _check(load_library().kf_admit(ctx, n, _ptr(slots), _ptr(tokens), _ptr(lens)), ctx)
+
+
 def kf_debug_logits(ctx, out):
     _check(load_library().kf_debug_logits(ctx, _ptr(out)), ctx)
 
@@ -215,6 +225,24 @@ class Decoder:
             out = np.zeros((self.B, max(k, 1)), np.int32)
         kf_decode_step(self.ctx, self.B, k, noise, out)
         return out
+
+    def teacher_step(self, k: int, noise, out=None):
+        """k AR steps in one call (the G* teacher); noise [B, k]; returns [B, k]."""
+        if out is None:
+            out = np.zeros((self.B, k), np.int32)
+        kf_teacher_step(self.ctx, self.B, k, noise, out)
+        return out
+
+    def admit(self, slots, prompts):
+        """Replace the sequences `slots` (an int or a list) by new prompts at a
+        step boundary."""
+        if np.isscalar(slots):
+            slots, prompts = [slots], [prompts]
+        sl = np.asarray(slots, np.int32)
+        lens = np.array([len(p) for p in prompts], np.int32)
+        toks = np.concatenate([np.asarray(p, np.int32) for p in prompts]) if len(prompts) else \
+            np.zeros(0, np.int32)
+        kf_admit(self.ctx, len(sl), sl, np.ascontiguousarray(toks), lens)
 
     def logits(self, nout: int):
         out = np.zeros((self.B, nout, self.model.vocab), np.float32)

@@ -28,6 +28,7 @@ SEED_WEIGHTS = 0
 SEED_PROMPTS = 1
 SEED_NOISE = 2
 SEED_LENGTHS = 3
+SEED_REQUESTS = 4
 
 
 @dataclass(frozen=True)
@@ -177,6 +178,18 @@ def make_noise(n_steps: int, batch: int, k: int,
     """fp32 U[0,1) noise, shape [n_steps, batch, max(k, 1)]."""
     rng = np.random.default_rng(seed)
     return rng.random((n_steps, batch, max(k, 1)), dtype=np.float32)
+
+
+def make_requests(n: int, prompt_len: int, gen_lo: int, gen_hi: int, k: int, vocab: int,
+                  seed: int = SEED_REQUESTS) -> list:
+    """Serving requests: (prompt of uniform ids, generation length uniform in
+    [gen_lo, gen_hi] rounded down to a multiple of k)."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        g = int(rng.integers(gen_lo, gen_hi + 1)) // k * k
+        out.append((rng.integers(0, vocab, size=prompt_len).astype(np.int32), max(k, g)))
+    return out
 
 
 def workload_prompts(w: Workload, batch: int | None = None) -> list:

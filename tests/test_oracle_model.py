@@ -98,6 +98,39 @@ def test_gstar_with_model_equals_ar_steps(tiny):
     assert g == oracle.ar_sample(m, prompt, z)
 
 
+def test_admit_one_pending_equals_prefill(tiny):
+    """Admitting a prompt with one pending token reproduces its prefill state."""
+    m, cfg = tiny
+    p1, p2, q = (list(x) for x in _prompts(cfg, 3, 9))
+    a = oracle.OracleDecoder(m)
+    a.prefill([p1, p2])
+    b = oracle.OracleDecoder(m)
+    b.prefill([p1, q])
+    b.admit(1, p2, 1)
+    sa, sb = a.seqs[1], b.seqs[1]
+    assert sa["committed"] == sb["committed"] and sa["pending"] == sb["pending"]
+    for (ka, va), (kb, vb) in zip(sa["cache"], sb["cache"]):
+        np.testing.assert_array_equal(ka, kb)
+        np.testing.assert_array_equal(va, vb)
+
+
+def test_admit_pending_tail_equals_cache_free_forward(tiny):
+    """A sequence admitted with P pending tokens, stepped once with k noise
+    slots, gives the tokens of the cache-free forward over the whole prompt
+    plus the noise rows (Alg. 1's first step)."""
+    m, cfg = tiny
+    p1, p2 = (list(x) for x in _prompts(cfg, 2, 11))
+    dec = oracle.OracleDecoder(m)
+    dec.prefill([p1, p1])
+    k, P = 3, 4
+    dec.admit(0, p2, P)
+    z = np.array([[0.21, 0.67, 0.93], [0.5, 0.5, 0.5]], np.float32)
+    toks = dec.step(k, z)
+    lg = oracle.full_forward_logits(m, p2, z[0], k)
+    want = [oracle.token_map(cfg, lg[j], z[0, j], np.float32) for j in range(k)]
+    assert [int(t) for t in toks[0]] == want
+
+
 def test_map_histogram_matches_softmax(tiny):
     from scipy import stats
     m, cfg = tiny
