@@ -15,6 +15,8 @@ Contents
   model.py  the push-forward causal Transformer (Sec. 3.3, Table 4) and the
             KV-cached decode of Alg. 1 (App. C.1), plus cache-free
             definitions (whole-sequence forward, textbook AR sampling).
+  train_attention.py  the SingleForward / DoubleForward training masks
+            (App. C.2) and dense masked attention over them.
 
 Pins (``tests/test_oracle_*.py``, run with ``-m "not gpu"``) tie each part
 to something other than itself: the worked example of App. B, a chi-square
