@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--gen", type=int, default=0, help="tokens per sequence (0: workload)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--no-ar", action="store_true", help="skip the k=1 AR leg")
+    p.add_argument("--train-attention", action="store_true",
+                   help="SingleForward / DoubleForward training attention (App. C.2)")
     p.add_argument("--serving", action="store_true",
                    help="the G* teacher call and continuous batching (LM1B, batch 64)")
     p.add_argument("--sweep-only", default="",
@@ -459,12 +461,67 @@ def run_serving(args):
     return 0
 
 
+def run_train_attention(args):
+    """SingleForward / DoubleForward attention (App. C.2), bf16, head_dim 64:
+    the mask-aware kernel against the same kernel visiting every key tile
+    (the dense-mask cost).  Reports TFLOP/s over the mask's pairs
+    (4 * 64 flops per visible (query, key) pair)."""
+    import ctypes
+    import torch
+    from paper_2606_10820_gb300 import build as kbuild
+    from paper_2606_10820_gb300 import kforcing as kf
+    kbuild.build()
+    lib = kf.load_library()
+    lib.kf_op_train_attention.argtypes = [ctypes.c_int32] * 7 + [ctypes.c_void_p] * 4 + \
+        [ctypes.c_int32, ctypes.c_void_p]
+    pk, peak_src = peaks()
+    for blocks, B, H, N, k in [(1, 32, 12, 128, 4), (1, 4, 12, 1024, 4), (2, 4, 12, 1024, 4),
+                               (1, 4, 12, 1024, 8)]:
+        T = N + blocks * N * k
+        g = torch.Generator(device="cuda").manual_seed(7)
+        q, kk, v = (torch.randn(B, T, H, 64, device="cuda", generator=g).to(torch.bfloat16) for _ in range(3))
+        out = torch.empty(B, T, H, 64, device="cuda")
+        # visible pairs: context rows, then per block row its context prefix and windows
+        ctx = N * (N + 1) // 2
+        pairs = ctx + k * ctx + N * k * (k + 1) // 2
+        if blocks == 2:
+            pairs += k * ctx + N * k * k + N * k * (k + 1) // 2
+        flops = 4.0 * 64 * pairs * B * H
+        res = {}
+        for dense in (0, 1):
+            def call():
+                lib.kf_op_train_attention(blocks, B, H, N, k, 0, T, q.data_ptr(), kk.data_ptr(),
+                                          v.data_ptr(), out.data_ptr(), dense, None)
+            for _ in range(max(3, args.warmup)):
+                call()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(max(10, args.steps)):
+                call()
+            e1.record()
+            torch.cuda.synchronize()
+            res[dense] = e0.elapsed_time(e1) / max(10, args.steps)
+        tf = flops / (res[0] / 1e3) / 1e12
+        print(json.dumps({
+            "metric": "training attention (App. C.2) TFLOP/s over the mask's pairs", "unit": "TFLOP/s",
+            "value": tf, "ms": res[0], "dense_mask_ms": res[1], "speedup_vs_dense_mask": res[1] / res[0],
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+                         "frac": tf / pk["bf16_tflops"], "peak_source": peak_src},
+            "config": {"mask": "SingleForward" if blocks == 1 else "DoubleForward", "batch": B, "heads": H,
+                       "N": N, "k": k, "tokens": T, "visible_pairs_per_head": pairs},
+            "data": "synthetic", "dtype": "bf16"}))
+    return 0
+
+
 def main():
     args = parse()
     if args.sweep:
         return run_sweep(args)
     if args.serving:
         return run_serving(args)
+    if args.train_attention:
+        return run_train_attention(args)
     if args.impl == "reference":
         return run_reference(args)
     import torch

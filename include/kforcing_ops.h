@@ -71,6 +71,35 @@ int kf_op_head_tokens_noalloc(int32_t rows, int32_t V, int32_t d, const void* x,
                               const void* w_head, const float* noise, float tau,
                               int32_t map_kind, int32_t* tokens, void* stream);
 
+/*
+ * Training-time attention of K-Forcing (App. C.2): SingleForward (blocks = 1)
+ * or DoubleForward (blocks = 2) in one call, for B sequences and H heads of
+ * head_dim 64.
+ *   Token layout of a sequence (T = N + blocks * N * k tokens): context
+ *   x_1..x_N at 0..N-1, then `blocks` blocks of N*k tokens, k per context
+ *   position; token (t, a) of block b (t = 0..N-1, a = 0..k-1) at
+ *   N + (b-1) N k + t k + a.  SingleForward's block 1 holds the noise
+ *   tokens; DoubleForward's blocks hold the first-round predictions
+ *   (Future-1) and the fresh noise (Future-2).
+ *   Mask: a context row i sees context keys 0..i; a block-1 row (t, a) sees
+ *   context 0..t and block-1 tokens (t, 0..a); a block-2 row (t, a) sees
+ *   context 0..t, all k block-1 tokens of window t and block-2 tokens
+ *   (t, 0..a) -- M_S and M_D of App. C.2.
+ * q, kk, v: [B][T][H][64] bf16, device, 16-byte aligned.  Queries are the rows
+ * [q_begin, q_end) of the layout (0..T for the whole mask; N + N k .. T for
+ * Future-2 alone, reusing the other rows' keys).  out: [B][q_end - q_begin][H][64]
+ * fp32, device, caller-owned.  Scale 1/sqrt(64), fp32 softmax, probabilities
+ * rounded to bf16 for the P.V product.
+ * dense = 0 visits only the key tiles a query tile can see (the context prefix
+ * and its windows: O(k) pairs relative to AR attention); dense = 1 visits every
+ * key tile with the same mask (the cost of a dense mask, for comparison).
+ * Errors: KF_E_ARG (sizes, ranges, alignment), KF_E_CUDA.  Asynchronous on
+ * `stream` (NULL: the default stream).
+ */
+int kf_op_train_attention(int32_t blocks, int32_t B, int32_t H, int32_t N, int32_t k,
+                          int32_t q_begin, int32_t q_end, const void* q, const void* kk,
+                          const void* v, float* out, int32_t dense, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,0 +1,98 @@
+"""kf_op_train_attention (SingleForward / DoubleForward, App. C.2) against the
+oracle's dense masked attention in fp64, through the C ABI (needs a GB300).
+
+Tolerance: the output rows are convex combinations of V rows; the kernel
+rounds the probabilities to bf16 for the P.V product (relative error <= 2^-9
+each, the row sums use the rounded values), so |out - ref| <= 2^-8 max|V| up
+to fp32 accumulation: the test allows 8e-3 max|V|.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+from oracle import train_attention as ta
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def env():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+    from paper_2606_10820_gb300 import kforcing as kf
+    lib = kf.load_library()
+    lib.kf_op_train_attention.argtypes = [ctypes.c_int32] * 7 + [ctypes.c_void_p] * 4 + \
+        [ctypes.c_int32, ctypes.c_void_p]
+    lib.kf_op_train_attention.restype = ctypes.c_int
+    return torch, lib
+
+
+def _run(torch, lib, blocks, B, H, N, k, q_begin=None, q_end=None, dense=0, seed=0):
+    T = N + blocks * N * k
+    q_begin = 0 if q_begin is None else q_begin
+    q_end = T if q_end is None else q_end
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    q, kk, v = ((torch.randn(B, T, H, 64, device="cuda", generator=g)).to(torch.bfloat16) for _ in range(3))
+    out = torch.full((B, q_end - q_begin, H, 64), float("nan"), device="cuda")
+    rc = lib.kf_op_train_attention(blocks, B, H, N, k, q_begin, q_end, q.data_ptr(), kk.data_ptr(),
+                                   v.data_ptr(), out.data_ptr(), dense, None)
+    assert rc == 0, rc
+    torch.cuda.synchronize()
+    return [x.float().cpu().numpy() for x in (q, kk, v)] + [out.cpu().numpy()]
+
+
+def _check(q, kk, v, out, blocks, N, k, q_begin, q_end):
+    mask = ta.mask_full(N, k, blocks)[q_begin:q_end]
+    for b in range(q.shape[0]):
+        ref = ta.masked_attention(q[b, q_begin:q_end], kk[b], v[b], mask)
+        err = np.abs(out[b] - ref).max()
+        assert err <= 8e-3 * np.abs(v[b]).max(), (b, err)
+
+
+CASES = [
+    (1, 2, 3, 5, 3), (1, 1, 2, 33, 4), (1, 1, 1, 130, 1), (1, 1, 2, 1, 8), (1, 1, 2, 70, 8),
+    (2, 2, 2, 9, 2), (2, 1, 3, 20, 4), (2, 1, 2, 7, 5), (2, 1, 1, 40, 3),
+]
+
+
+@pytest.mark.parametrize("blocks,B,H,N,k", CASES)
+@pytest.mark.parametrize("dense", [0, 1])
+def test_train_attention_matches_dense_oracle(env, blocks, B, H, N, k, dense):
+    torch, lib = env
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, dense=dense, seed=N * 31 + k)
+    assert np.isfinite(out).all()
+    _check(q, kk, v, out, blocks, N, k, 0, N + blocks * N * k)
+
+
+def test_double_future2_only_rows(env):
+    """DoubleForward with KV reuse: only the Future-2 queries."""
+    torch, lib = env
+    blocks, B, H, N, k = 2, 2, 2, 37, 4
+    qb, qe = N + N * k, N + 2 * N * k
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, qb, qe, seed=5)
+    _check(q, kk, v, out, blocks, N, k, qb, qe)
+
+
+def test_long_sequence_sampled_rows(env):
+    """N = 512, k = 4 (T = 2560): rows sampled across the blocks."""
+    torch, lib = env
+    blocks, B, H, N, k = 1, 1, 2, 512, 4
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, seed=9)
+    mask = ta.mask_single(N, k)
+    rows = np.array([0, 1, 127, 128, 511, N, N + 3, N + 4 * 200 + 2, N + 4 * 511 + 3])
+    ref = ta.masked_attention(q[0, rows], kk[0], v[0], mask[rows])
+    assert np.abs(out[0, rows] - ref).max() <= 8e-3 * np.abs(v[0]).max()
+
+
+def test_argument_errors(env):
+    torch, lib = env
+    buf = torch.zeros(64, dtype=torch.bfloat16, device="cuda")
+    out = torch.zeros(64, device="cuda")
+    p = buf.data_ptr()
+    for args in [(3, 1, 1, 4, 2, 0, 12), (1, 1, 1, 4, 2, 0, 13), (1, 1, 1, 4, 2, 5, 5),
+                 (1, 0, 1, 4, 2, 0, 12), (2, 1, 1, 4, 0, 0, 4)]:
+        assert lib.kf_op_train_attention(*args, p, p, p, out.data_ptr(), 0, None) == -1, args
