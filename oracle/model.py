@@ -41,9 +41,14 @@ class OracleModel:
         return h
 
     def noise_rows(self, z, pos) -> np.ndarray:
+        """Fully causal: one row per noise value.  Standard MTP (cfg.mtp_k > 0,
+        Sec. 3.3): the k values are one noise-conditioning token; reading: its
+        features are the k values' sinusoidal features concatenated."""
         cfg = self.cfg
         z = np.asarray(z, np.float32).astype(self.dtype)
         feat = ops.noise_features(z, cfg.tau, cfg.d_model, cfg.noise_scale)
+        if cfg.mtp_k:
+            feat = feat.reshape(1, -1)
         h = ops.noise_encoder(feat, self.w["ne_w1"], self.w["ne_b1"],
                               self.w["ne_w2"], self.w["ne_b2"])
         if cfg.pos == "learned":
@@ -88,6 +93,12 @@ class OracleModel:
         """Head(o): final RMSNorm, untied LM head, divided by tau."""
         o = ops.rmsnorm(h_rows, self.w["final_norm"], self.cfg.rms_eps)
         return (o @ self.w["w_head"].T) / self.cfg.tau
+
+    def logits_mtp(self, h_row) -> np.ndarray:
+        """The k independent MTP heads on the noise token's final hidden
+        state (Sec. 3.3): [k, V], head j = final RMSNorm then w_mtp[j], / tau."""
+        o = ops.rmsnorm(np.asarray(h_row).reshape(1, -1), self.w["final_norm"], self.cfg.rms_eps)
+        return np.stack([(o @ wj.T)[0] for wj in self.w["w_mtp"]]) / self.cfg.tau
 
     def empty_cache(self):
         z = np.zeros((0, self.H, self.hd), self.dtype)
@@ -161,7 +172,13 @@ class OracleDecoder:
             P = len(s["pending"])
             pos_x = np.arange(c, c + P)
             h = self.m.token_rows(s["pending"], pos_x)
-            if k > 0:
+            mtp = cfg.mtp_k > 0 and k > 0
+            if mtp:
+                assert k == cfg.mtp_k
+                pos_z = np.array([c + P])
+                h = np.concatenate([h, self.m.noise_rows(z[b, :k], pos_z)], 0)
+                pos = np.concatenate([pos_x, pos_z])
+            elif k > 0:
                 pos_z = np.arange(c + P, c + P + k)
                 h = np.concatenate([h, self.m.noise_rows(z[b, :k], pos_z)], 0)
                 pos = np.concatenate([pos_x, pos_z])
@@ -172,8 +189,11 @@ class OracleDecoder:
             # C <- [C; C_x]: keep the P context rows' KV, discard the noise KV
             s["cache"] = [(np.concatenate([ck, nk[:P]]), np.concatenate([cv, nv[:P]]))
                           for (ck, cv), (nk, nv) in zip(s["cache"], new)]
-            head_rows = o[P:] if k > 0 else o[P - 1:P]
-            lg = self.m.logits(head_rows)
+            if mtp:
+                lg = self.m.logits_mtp(o[P])
+            else:
+                head_rows = o[P:] if k > 0 else o[P - 1:P]
+                lg = self.m.logits(head_rows)
             for j in range(nout):
                 toks[b, j] = token_map(cfg, lg[j], z[b, j], self.map_dtype)
             if want_logits:

@@ -49,6 +49,8 @@ class ModelConfig:
     rope_theta: float = 10000.0
     noise_scale: float = 1000.0
     map: str = "icdf"          # "icdf" | "argmax"
+    mtp_k: int = 0             # 0: fully causal (k noise tokens, shared head);
+                               # > 0: standard MTP (Sec. 3.3): one noise token, mtp_k heads
 
     @property
     def head_dim(self) -> int:
@@ -84,6 +86,10 @@ OWT = ModelConfig(n_layer=12, d_model=768, n_head=12, d_ff=3072, vocab=50257,
                   max_len=1024, pos="rope", dtype="bf16")
 MEDIUM = ModelConfig(n_layer=24, d_model=1024, n_head=16, d_ff=4096,
                      vocab=50257, max_len=2048, pos="rope", dtype="bf16")
+
+# standard-MTP variants of the same backbones (the architecture ablation of Sec. 3.3)
+TINY_MTP = TINY.replace(mtp_k=3)
+LM1B_MTP = LM1B.replace(mtp_k=4)
 
 WORKLOADS = {
     # tiny fp32 parity case: one k=2 step after a 32-token prompt
@@ -126,13 +132,15 @@ def weight_shapes(cfg: ModelConfig) -> dict:
         "w_down": (L, d, F),
         "final_norm": (d,),
         "w_head": (V, d),
-        "ne_w1": (h, d),
+        "ne_w1": (h, d * max(1, cfg.mtp_k)),
         "ne_b1": (h,),
         "ne_w2": (d, h),
         "ne_b2": (d,),
     }
     if cfg.pos == "learned":
         shapes["pos_emb"] = (cfg.max_len, d)
+    if cfg.mtp_k:
+        shapes["w_mtp"] = (cfg.mtp_k, V, d)
     return shapes
 
 

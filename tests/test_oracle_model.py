@@ -131,6 +131,47 @@ def test_admit_pending_tail_equals_cache_free_forward(tiny):
     assert [int(t) for t in toks[0]] == want
 
 
+def test_mtp_with_one_head_equals_fully_causal_k1():
+    """Standard MTP with k = 1, its head equal to the shared head, is the
+    fully causal step with one noise token (both are one noise row decoded
+    by the same head)."""
+    from synth import TINY
+    cfg1 = TINY.replace(mtp_k=1)
+    w1 = make_weights(cfg1)
+    w0 = {n: a for n, a in w1.items() if n != "w_mtp"}
+    w1["w_mtp"] = w1["w_head"][None].copy()
+    prompts = make_prompts([7, 10], cfg1.vocab)
+    a = oracle.OracleDecoder(oracle.OracleModel(cfg1, w1))
+    b = oracle.OracleDecoder(oracle.OracleModel(TINY, w0))
+    a.prefill(prompts)
+    b.prefill(prompts)
+    for z in ([[0.3], [0.9]], [[0.05], [0.61]]):
+        z = np.array(z, np.float32)
+        ta, la = a.step(1, z, want_logits=True)
+        tb, lb = b.step(1, z, want_logits=True)
+        np.testing.assert_array_equal(ta, tb)
+        np.testing.assert_allclose(la, lb, rtol=0, atol=1e-12)
+
+
+def test_mtp_step_equals_cache_free_forward():
+    """An MTP step after prefill gives the heads' maps of the cache-free
+    forward over the whole prompt plus the one noise token."""
+    from synth import TINY_MTP as cfg
+    w = make_weights(cfg)
+    m = oracle.OracleModel(cfg, w)
+    p = list(make_prompts([9], cfg.vocab)[0])
+    dec = oracle.OracleDecoder(m)
+    dec.prefill([p])
+    z = np.array([[0.14, 0.52, 0.97]], np.float32)
+    toks = dec.step(3, z)
+    n = len(p)
+    h = np.concatenate([m.token_rows(p, np.arange(n)), m.noise_rows(z[0], np.array([n]))], 0)
+    o, _ = m.forward(h, np.arange(n + 1), m.empty_cache())
+    lg = m.logits_mtp(o[n])
+    want = [oracle.token_map(cfg, lg[j], z[0, j], np.float32) for j in range(3)]
+    assert [int(t) for t in toks[0]] == want
+
+
 def test_map_histogram_matches_softmax(tiny):
     from scipy import stats
     m, cfg = tiny
