@@ -96,20 +96,24 @@ def kind_costs(model, B, P, k, ctx_lens):
     d, F, V, H = model.d_model, model.d_ff, model.vocab, model.n_head
     hd = d // H
     e = 2 if model.dtype == "bf16" else 4
-    R = B * (P + k)
+    kz = 1 if (getattr(model, "mtp_k", 0) and k) else k     # noise rows per sequence
+    R = B * (P + kz)
     nh = B * max(k, 1)
     nchunk = -(-V // 32)
 
     def gemm(M, N, K, out_bytes):
         return {"bytes": N * K * e + M * K * e + out_bytes, "flops": 2.0 * M * N * K}
-    keys = sum(int(c) + P + k for c in ctx_lens)
-    vis = sum(sum(int(c) + i + 1 for i in range(P + k)) for c in ctx_lens)
+    keys = sum(int(c) + P + kz for c in ctx_lens)
+    vis = sum(sum(int(c) + i + 1 for i in range(P + kz)) for c in ctx_lens)
+    head = gemm(nh, V, d, nh * nchunk * 16)
+    if kz != k:        # MTP: k heads over B rows
+        head = {"bytes": k * V * d * e + B * d * e + nh * nchunk * 16, "flops": 2.0 * nh * V * d}
     return {
         "gemm_qkv": gemm(R, 3 * d, d, R * 3 * d * e),
         "gemm_o": gemm(R, d, d, 2 * R * d * 4),
         "gemm_up": gemm(R, F, d, R * F * e),
         "gemm_down": gemm(R, d, F, 2 * R * d * 4),
-        "gemm_head": gemm(nh, V, d, nh * nchunk * 16),
+        "gemm_head": head,
         "attention": {"bytes": keys * H * hd * 2 * e + R * d * 4 + R * d * e,
                       "flops": 4.0 * vis * H * hd},
     }
@@ -119,13 +123,18 @@ def step_bytes_flops(model, B, P, k, ctx_lens):
     """Algorithmic bytes/flops of one decode call (weights once, KV once)."""
     d, F, V, L, H = model.d_model, model.d_ff, model.vocab, model.n_layer, model.n_head
     e = 2 if model.dtype == "bf16" else 4
-    w = L * (4 * d * d + 2 * d * F) * e + V * d * e + (2 * model.ne_hidden * d * e if k else 0)
+    mtp = bool(getattr(model, "mtp_k", 0) and k)
+    kz = 1 if mtp else k                           # noise rows per sequence
+    ne_in = k * d if mtp else d                    # NoiseEnc input width
+    heads = k if mtp else 1
+    w = L * (4 * d * d + 2 * d * F) * e + heads * V * d * e + \
+        ((model.ne_hidden * ne_in + model.ne_hidden * d) * e if k else 0)
     kv_tok = 2 * L * d * e
-    byt = w + sum(int(c) for c in ctx_lens) * kv_tok + B * (P + k) * kv_tok
-    R = B * (P + k)
+    byt = w + sum(int(c) for c in ctx_lens) * kv_tok + B * (P + kz) * kv_tok
+    R = B * (P + kz)
     fl = 2.0 * R * L * (4 * d * d + 2 * d * F) + 2.0 * B * max(k, 1) * V * d + \
-        (4.0 * B * k * model.ne_hidden * d if k else 0) + \
-        4.0 * L * d * sum(sum(int(c) + i + 1 for i in range(P + k)) for c in ctx_lens)
+        (2.0 * B * kz * model.ne_hidden * (ne_in + d) if k else 0) + \
+        4.0 * L * d * sum(sum(int(c) + i + 1 for i in range(P + kz)) for c in ctx_lens)
     return byt, fl
 
 
@@ -278,6 +287,7 @@ SWEEP = [  # (workload, batch, ks) -- the non-headline configurations
     ("owt", 128, (4, 2, 1)), ("owt", 256, (4, 2, 1)),
     ("owt_paged", 512, (4, 1)),
     ("medium", 256, (8, 4, 1)),
+    ("lm1b_mtp", 64, (4, 1)),
 ]
 
 

@@ -83,6 +83,13 @@ typedef struct kf_config {
   float rms_eps;        /* RMSNorm epsilon                                    */
   float rope_theta;     /* RoPE base                                          */
   float noise_scale;    /* sinusoid argument = noise_scale * z                */
+  int32_t mtp_k;        /* 0: the fully causal model (k noise tokens, one
+                           shared head); > 0: the standard MTP variant (Sec.
+                           3.3) with mtp_k heads: a k-step (k = mtp_k) feeds
+                           one noise-conditioning token whose NoiseEnc input
+                           is the k values' sinusoidal features concatenated
+                           (k * d wide), and head j maps its hidden state
+                           with noise[b][j].  mtp_k <= max_k.               */
 } kf_config;
 
 /*
@@ -102,10 +109,11 @@ typedef struct kf_weights {
   const float* w_down;      /* [L][d][F]                               */
   const float* final_norm;  /* [d]                                     */
   const float* w_head;      /* [V][d] (untied)                         */
-  const float* ne_w1;       /* [noise_hidden][d]                       */
+  const float* ne_w1;       /* [noise_hidden][d] ([noise_hidden][mtp_k d] for MTP) */
   const float* ne_b1;       /* [noise_hidden]                          */
   const float* ne_w2;       /* [d][noise_hidden]                       */
   const float* ne_b2;       /* [d]                                     */
+  const float* w_mtp;       /* [mtp_k][V][d], the MTP heads; NULL unless mtp_k > 0 */
 } kf_weights;
 
 typedef struct kf_ctx kf_ctx;
@@ -137,6 +145,9 @@ int kf_prefill(kf_ctx* ctx, int32_t B, const int32_t* tokens,
  *           its logits with noise[b][j].  Emits k tokens per sequence.
  *   k == 0: the AR teacher step (Eq. 1 with one token): the last pending
  *           row's logits mapped with noise[b][0].  Emits 1 token.
+ *   MTP models (mtp_k > 0): k must be 0 or mtp_k; the k-step feeds the P
+ *           pending tokens and one noise token, and head j maps the noise
+ *           token's hidden state with noise[b][j].  Emits k tokens.
  * noise:      [B][max(k,1)] fp32 in [0,1), host or device.
  * out_tokens: [B][max(k,1)] int32, host or device, caller-owned.
  * Afterwards each sequence's cache holds P more tokens and the emitted tokens

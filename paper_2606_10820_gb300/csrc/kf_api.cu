@@ -47,6 +47,9 @@ struct kf_ctx {
   std::vector<LayerW> layers;
   float* final_norm = nullptr;
   void* w_head = nullptr;
+  void* w_mtp = nullptr;        // [mtp_k][V_pad][d] MTP heads (mtp_k > 0)
+  int mtp_k = 0;
+  bool last_mtp = false;        // the last step decoded with the MTP heads
   void* ne_w1 = nullptr;
   float* ne_b1 = nullptr;
   void* ne_w2 = nullptr;
@@ -294,12 +297,16 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   cudaStream_t s = c->stream;
   PdlScope pdl(!c->prof && !(c->cfg.flags & KF_FLAG_NO_PDL));
   const int d = c->d;
-  const int S = P + k, R = B * S, nout = k > 0 ? k : 1, nh = B * nout;
+  // standard MTP (Sec. 3.3): one noise-conditioning token per sequence whose
+  // NoiseEnc input is the k values' features side by side; k heads decode it
+  const bool mtp = c->mtp_k > 0 && k > 0;
+  const int kz = mtp ? 1 : k;                      // noise rows per sequence
+  const int S = P + kz, R = B * S, nout = k > 0 ? k : 1, nh = mtp ? B : B * nout;
   prof_begin(c, KF_KIND_ROWMAP);
-  launch_rowmap(B, P, k, c->d_len, c->row_seq, c->row_pos, c->noise_map, c->head_map, s);
+  launch_rowmap(B, P, kz, c->d_len, c->row_seq, c->row_pos, c->noise_map, c->head_map, s);
   prof_end(c);
   prof_begin(c, KF_KIND_EMBED);
-  launch_embed_pending(c->bf16, B, P, k, c->d_pending, c->pend_stride, c->tok_emb, c->pos_emb,
+  launch_embed_pending(c->bf16, B, P, kz, c->d_pending, c->pend_stride, c->tok_emb, c->pos_emb,
                        c->row_pos, c->V, d, c->x, c->fused ? c->xn : nullptr,
                        c->fused ? c->ss : nullptr, c->d_err, s);
   if (k > 0)
@@ -308,26 +315,40 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   prof_end(c);
   if (k > 0) {
     // h_z = NoiseEnc(z): W2 . gelu(W1 s(z, tau) + b1) + b2, written into the noise rows
+    // (MTP: the B rows of k * d features, [B][k][d] as laid out by the feature kernel)
+    const int ne_in = mtp ? k * d : d;
     Epi e1;
     e1.kind = EPI_BIAS_GELU; e1.out = c->nhid; e1.ldo = c->NH; e1.bias = c->ne_b1;
-    gemm(c, KF_KIND_NOISE_GEMM, B * k, c->NH, d, c->nfeat, d, c->ne_w1, d, e1);
+    gemm(c, KF_KIND_NOISE_GEMM, B * kz, c->NH, ne_in, c->nfeat, ne_in, c->ne_w1, ne_in, e1);
     Epi e2;
     e2.kind = EPI_NOISE_OUT; e2.x = c->x; e2.ldx = d; e2.bias = c->ne_b2;
     e2.row_map = c->noise_map; e2.row_pos = c->row_pos; e2.pos_emb = c->pos_emb;
     if (c->fused) { e2.xb_out = c->xn; e2.ss_out = c->ss; e2.nslot = d / 64; }
-    gemm(c, KF_KIND_NOISE_GEMM, B * k, d, c->NH, c->nhid, c->NH, c->ne_w2, c->NH, e2);
+    gemm(c, KF_KIND_NOISE_GEMM, B * kz, d, c->NH, c->nhid, c->NH, c->ne_w2, c->NH, e2);
   }
   enqueue_layers(c, R, B, nullptr, S);
   prof_begin(c, KF_KIND_HEAD_NORM);
   launch_rmsnorm(c->bf16, nh, c->head_map, c->x, d, c->final_norm, c->cfg.rms_eps, c->head_in, s);
   prof_end(c);
-  Epi eh;
-  eh.kind = EPI_HEAD; eh.inv_tau = 1.0f / c->cfg.tau; eh.n_valid = c->V; eh.rec = c->rec;
-  eh.nchunk = c->nchunk;
-  gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, d, c->head_in, d, c->w_head, d, eh);
+  if (mtp) {
+    // head j over the B noise rows; its chunk records at rows j * B + b
+    for (int j = 0; j < k; ++j) {
+      Epi eh;
+      eh.kind = EPI_HEAD; eh.inv_tau = 1.0f / c->cfg.tau; eh.n_valid = c->V;
+      eh.rec = c->rec + (size_t)j * B * c->nchunk; eh.nchunk = c->nchunk;
+      gemm(c, KF_KIND_GEMM_HEAD, B, c->V_pad, d, c->head_in, d,
+           static_cast<const char*>(c->w_mtp) + (size_t)j * c->V_pad * d * c->esz, d, eh);
+    }
+  } else {
+    Epi eh;
+    eh.kind = EPI_HEAD; eh.inv_tau = 1.0f / c->cfg.tau; eh.n_valid = c->V; eh.rec = c->rec;
+    eh.nchunk = c->nchunk;
+    gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, d, c->head_in, d, c->w_head, d, eh);
+  }
   prof_begin(c, KF_KIND_HEAD_SELECT);
-  launch_head_select(c->bf16, nh, c->rec, c->nchunk, c->head_in, d, c->w_head, c->V,
-                     1.0f / c->cfg.tau, c->cfg.map_kind, noise, c->tokens, s);
+  launch_head_select(c->bf16, B * nout, c->rec, c->nchunk, c->head_in, d, mtp ? c->w_mtp : c->w_head,
+                     c->V, 1.0f / c->cfg.tau, c->cfg.map_kind, noise, c->tokens, mtp ? B : 0,
+                     (size_t)c->V_pad * d, s);
   prof_end(c);
   prof_begin(c, KF_KIND_COMMIT);
   launch_commit(B, P, k, c->tokens, c->d_pending, c->pend_stride, c->d_len, s);
@@ -393,6 +414,8 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
   else if (!(cfg.tau > 0.f)) bad = "tau must be > 0";
   else if (!(cfg.rms_eps >= 0.f)) bad = "rms_eps must be >= 0";
   else if (cfg.n_pages < 0 || cfg.prefill_rows < 16) bad = "bad n_pages / prefill_rows";
+  else if (cfg.mtp_k < 0 || cfg.mtp_k > cfg.max_k) bad = "mtp_k must be in 0..max_k";
+  else if (cfg.mtp_k > 0 && !w->w_mtp) bad = "w_mtp is NULL with mtp_k > 0";
   else if (!w->tok_emb || !w->attn_norm || !w->wqkv || !w->wo || !w->mlp_norm || !w->w_up ||
            !w->w_down || !w->final_norm || !w->w_head || !w->ne_w1 || !w->ne_b1 || !w->ne_w2 ||
            !w->ne_b2)
@@ -427,13 +450,15 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
   c->esz = c->bf16 ? 2 : 4;
   c->d = cfg.d_model; c->H = cfg.n_head; c->hd = cfg.d_model / cfg.n_head; c->L = cfg.n_layer; c->F = cfg.d_ff; c->V = cfg.vocab;
   c->NH = cfg.noise_hidden; c->V_pad = round_up(cfg.vocab, 256); c->max_k = cfg.max_k;
+  c->mtp_k = cfg.mtp_k;
   c->nchunk = ceil_div(cfg.vocab, kChunk);
   const int d = c->d, L = c->L, F = c->F, V = c->V, NH = c->NH;
   const bool dev_w = is_device_ptr(w->tok_emb);
 
   // -- weights: staged through one fp32 device buffer, converted to storage type
+  const int ne_in = d * std::max(1, cfg.mtp_k);   // NoiseEnc input width
   size_t max_elems = std::max({(size_t)V * d, (size_t)L * 3 * d * d, (size_t)L * F * d,
-                               (size_t)NH * d, (size_t)cfg.max_len * d});
+                               (size_t)NH * ne_in, (size_t)cfg.max_len * d});
   float* stage = nullptr;
   if ((r = dalloc(c, &stage, max_elems * 4, false))) return bail(r);
   const float* fold_gain = nullptr;   // gains to fold into the columns being uploaded
@@ -482,11 +507,19 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
       (r = fbuf(&c->final_norm, d)) || (r = upload(w->final_norm, d, c->final_norm, false)) ||
       (r = wbuf(&c->w_head, (size_t)c->V_pad * d)) ||
       (r = upload(w->w_head, (size_t)V * d, c->w_head, true)) ||
-      (r = wbuf(&c->ne_w1, (size_t)NH * d)) || (r = upload(w->ne_w1, (size_t)NH * d, c->ne_w1, true)) ||
+      (r = wbuf(&c->ne_w1, (size_t)NH * ne_in)) || (r = upload(w->ne_w1, (size_t)NH * ne_in, c->ne_w1, true)) ||
       (r = fbuf(&c->ne_b1, NH)) || (r = upload(w->ne_b1, NH, c->ne_b1, false)) ||
       (r = wbuf(&c->ne_w2, (size_t)d * NH)) || (r = upload(w->ne_w2, (size_t)d * NH, c->ne_w2, true)) ||
       (r = fbuf(&c->ne_b2, d)) || (r = upload(w->ne_b2, d, c->ne_b2, false)))
     return bail(r);
+  if (c->mtp_k > 0) {
+    // MTP heads, each padded to V_pad zero rows like w_head
+    if ((r = wbuf(&c->w_mtp, (size_t)c->mtp_k * c->V_pad * d))) return bail(r);
+    for (int j = 0; j < c->mtp_k; ++j)
+      if ((r = upload(w->w_mtp + (size_t)j * V * d, (size_t)V * d,
+                      static_cast<char*>(c->w_mtp) + (size_t)j * c->V_pad * d * c->esz, true)))
+        return bail(r);
+  }
   for (int l = 0; l < L; ++l) {
     LayerW lw;
     lw.wqkv = (char*)wqkv + (size_t)l * 3 * d * d * c->esz;
@@ -811,6 +844,7 @@ int kf_teacher_step(kf_ctx* c, int32_t B, int32_t k, const float* noise, int32_t
   for (int b = 0; b < B; ++b) c->h_len[b] += P + k - 1;
   c->P = 1;
   c->last_nh = B;
+  c->last_mtp = false;
   c->have_step = true;
   if (!is_device_ptr(out_tokens)) {
     KF_CUDA(cudaStreamSynchronize(c->stream));
@@ -827,6 +861,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
   if (!c->have_batch) return fail(c, KF_E_STATE, "decode before prefill");
   if (B != c->B) return fail(c, KF_E_ARG, "B differs from the prefilled batch");
   if (k < 0 || k > c->max_k) return fail(c, KF_E_ARG, "k out of range 0..max_k");
+  if (c->mtp_k > 0 && k > 0 && k != c->mtp_k) return fail(c, KF_E_ARG, "an MTP model steps with k = 0 or mtp_k");
   if (!noise || !out_tokens) return fail(c, KF_E_ARG, "noise or out_tokens is NULL");
   const int P = c->P, nout = k > 0 ? k : 1;
   for (int b = 0; b < B; ++b)
@@ -877,6 +912,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
   for (int b = 0; b < B; ++b) c->h_len[b] += P;
   c->P = nout;
   c->last_nh = B * nout;
+  c->last_mtp = c->mtp_k > 0 && k > 0;
   c->have_step = true;
   if (!is_device_ptr(out_tokens)) {
     KF_CUDA(cudaStreamSynchronize(c->stream));
@@ -921,9 +957,21 @@ int kf_debug_logits(kf_ctx* c, float* out) {
     KF_CUDA(cudaMalloc(&tmp, (size_t)nh * c->V * 4));
     dst = tmp;
   }
-  Epi e;
-  e.kind = EPI_LOGITS; e.outf = dst; e.ldo = c->V; e.inv_tau = 1.0f / c->cfg.tau; e.n_valid = c->V;
-  gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, c->d, c->head_in, c->d, c->w_head, c->d, e);
+  if (c->last_mtp) {
+    // head j of the B noise rows -> out[b][j][V]
+    const int kk = nh / c->B;
+    for (int j = 0; j < kk; ++j) {
+      Epi e;
+      e.kind = EPI_LOGITS; e.outf = dst + (size_t)j * c->V; e.ldo = kk * c->V;
+      e.inv_tau = 1.0f / c->cfg.tau; e.n_valid = c->V;
+      gemm(c, KF_KIND_GEMM_HEAD, c->B, c->V_pad, c->d, c->head_in, c->d,
+           static_cast<const char*>(c->w_mtp) + (size_t)j * c->V_pad * c->d * c->esz, c->d, e);
+    }
+  } else {
+    Epi e;
+    e.kind = EPI_LOGITS; e.outf = dst; e.ldo = c->V; e.inv_tau = 1.0f / c->cfg.tau; e.n_valid = c->V;
+    gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, c->d, c->head_in, c->d, c->w_head, c->d, e);
+  }
   cudaError_t err = cudaGetLastError();
   if (err == cudaSuccess && !dev)
     err = cudaMemcpyAsync(out, tmp, (size_t)nh * c->V * 4, cudaMemcpyDeviceToHost, c->stream);

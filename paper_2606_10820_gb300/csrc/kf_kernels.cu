@@ -322,11 +322,23 @@ __device__ __forceinline__ void ld_vec(const __nv_bfloat16* p, float* o) {
 template <typename TA>
 __global__ void __launch_bounds__(kSelThreads)
 k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
-              const TA* __restrict__ w_head, int V, float inv_tau, int map_kind,
-              const float* __restrict__ noise, int32_t* __restrict__ tokens) {
+              const TA* __restrict__ w_head_all, int V, float inv_tau, int map_kind,
+              const float* __restrict__ noise, int32_t* __restrict__ tokens, int mtp_rows,
+              size_t head_stride) {
   pdl_trigger();
   pdl_wait();
+  // one block per mapped row; MTP (mtp_rows = B > 0): block j B + b is head j
+  // of sequence b (records in that order), hidden row b, weights w_head + j
+  // head_stride, noise and token index b k + j
   const int row = blockIdx.x;
+  int hrow = row, zrow = row;
+  const TA* w_head = w_head_all;
+  if (mtp_rows > 0) {
+    const int b = row % mtp_rows, j = row / mtp_rows, kk = gridDim.x / mtp_rows;
+    hrow = b;
+    zrow = b * kk + j;
+    w_head = w_head_all + (size_t)j * head_stride;
+  }
   const HeadRec* rec = rec_all + (size_t)row * nchunk;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   __shared__ float s_red[kSelThreads / 32];
@@ -381,7 +393,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   }
   __syncthreads();
   if (map_kind == KF_MAP_ARGMAX) {
-    if (t == 0) tokens[row] = s_redi[0];
+    if (t == 0) tokens[zrow] = s_redi[0];
     return;
   }
   const float M = s_M;
@@ -418,7 +430,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
       run += s_red[w];
     }
     s_wexcl[kSelThreads / 32] = run;     // S
-    s_T = noise[row] * run;
+    s_T = noise[zrow] * run;
     s_redi[2] = kSelThreads;             // first crossing thread (none yet)
   }
   __syncthreads();
@@ -462,7 +474,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   const int cstar = s_chunk;
   {
     // the warp's NQ ids side by side, so their weight loads are in flight together
-    const TA* hr = head_in + (size_t)row * d;
+    const TA* hr = head_in + (size_t)hrow * d;
     constexpr int VEC = 16 / sizeof(TA);
     constexpr int NQ = kChunk / (kSelThreads / 32);
     const int jj0 = warp * NQ;
@@ -511,21 +523,22 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
     if (hit) tok = cstar * kChunk + (__ffs(hit) - 1);
     else if (pos) tok = cstar * kChunk + (31 - __clz(pos));
     else tok = min(V - 1, cstar * kChunk + 31);
-    tokens[row] = tok;
+    tokens[zrow] = tok;
   }
 }
 
 void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
                         int d, const void* w_head, int V, float inv_tau, int map_kind,
-                        const float* noise, int32_t* tokens, cudaStream_t s) {
+                        const float* noise, int32_t* tokens, int mtp_rows, size_t head_stride,
+                        cudaStream_t s) {
   if (n_rows == 0) return;
   if (bf16)
     kf_launch(k_head_select<__nv_bfloat16>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk,
         (const __nv_bfloat16*)head_in, d, (const __nv_bfloat16*)w_head, V, inv_tau, map_kind,
-        noise, tokens);
+        noise, tokens, mtp_rows, head_stride);
   else
     kf_launch(k_head_select<float>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk, (const float*)head_in, d,
-        (const float*)w_head, V, inv_tau, map_kind, noise, tokens);
+        (const float*)w_head, V, inv_tau, map_kind, noise, tokens, mtp_rows, head_stride);
 }
 
 // ---------------------------------------------------------------- commit

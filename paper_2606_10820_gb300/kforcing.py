@@ -44,11 +44,11 @@ class kf_config(ctypes.Structure):
         "n_layer", "d_model", "n_head", "d_ff", "vocab", "max_len", "noise_hidden",
         "pos_kind", "dtype", "map_kind", "max_batch", "max_k", "page_size", "n_pages",
         "prefill_rows", "flags")] + [(n, ctypes.c_float) for n in (
-        "tau", "rms_eps", "rope_theta", "noise_scale")]
+        "tau", "rms_eps", "rope_theta", "noise_scale")] + [("mtp_k", ctypes.c_int32)]
 
 
 WEIGHT_FIELDS = ("tok_emb", "pos_emb", "attn_norm", "wqkv", "wo", "mlp_norm", "w_up", "w_down",
-                 "final_norm", "w_head", "ne_w1", "ne_b1", "ne_w2", "ne_b2")
+                 "final_norm", "w_head", "ne_w1", "ne_b1", "ne_w2", "ne_b2", "w_mtp")
 
 
 class kf_weights(ctypes.Structure):
@@ -126,6 +126,7 @@ def make_config(model, max_batch: int, max_k: int, n_pages: int = 0, flags: int 
     c.prefill_rows, c.flags = prefill_rows, flags
     c.tau, c.rms_eps, c.rope_theta, c.noise_scale = (model.tau, model.rms_eps, model.rope_theta,
                                                      model.noise_scale)
+    c.mtp_k = getattr(model, "mtp_k", 0)
     return c
 
 

@@ -103,6 +103,9 @@ WORKLOADS = {
     # OWT-shaped high-load paged serving: ragged prompts in [128, 896], 128 new
     "owt_paged": Workload("owt_paged", OWT, batch=512, prompt_len=0,
                           gen_len=128, ks=(4, 1), ragged=(128, 896)),
+    # the standard-MTP variant of the LM1B-shaped model (Sec. 3.3 ablation)
+    "lm1b_mtp": Workload("lm1b_mtp", LM1B_MTP, batch=64, prompt_len=32, gen_len=96,
+                         ks=(4, 1)),
     # medium stress shape: prompt 1024 -> 2048
     "medium": Workload("medium", MEDIUM, batch=256, prompt_len=1024,
                        gen_len=1024, ks=(8, 4, 1)),

@@ -53,9 +53,9 @@ def test_binding_uses_the_c_names(lib):
 
 def test_struct_layout_matches_header():
     from paper_2606_10820_gb300 import kforcing as kf
-    # 16 int32 fields followed by 4 floats; 14 pointers
-    assert ctypes.sizeof(kf.kf_config) == 20 * 4
-    assert ctypes.sizeof(kf.kf_weights) == 14 * ctypes.sizeof(ctypes.c_void_p)
+    # 16 int32 fields, 4 floats, then mtp_k; 15 pointers
+    assert ctypes.sizeof(kf.kf_config) == 21 * 4
+    assert ctypes.sizeof(kf.kf_weights) == 15 * ctypes.sizeof(ctypes.c_void_p)
 
 
 def test_init_rejects_bad_config_on_host(lib):
