@@ -11,18 +11,19 @@
 // SingleForward is blocks = 1 (block 1 = the noise tokens); DoubleForward is
 // blocks = 2 (Future-1 predictions, Future-2 noise).
 //
-// A CTA (4 warps) takes 16 consecutive query rows of one (sequence, head)
-// and walks three disjoint key ranges: the context prefix up to the largest
-// context key any of its rows sees, and the block-1 / block-2 windows of its
-// rows' groups.  Each range goes in 128-key tiles (cp.async into swizzled
-// shared memory, double-buffered); inside a tile every (row, key) pair is
-// masked by the rule above, except in warps whose 32 keys are context keys
-// every row of the tile sees.  Per tile, warp w takes keys 32w..32w+31:
-// S = Q K^T and O += P V on mma.sync m16n8k16 with P in registers and an
-// online softmax per warp; the four warps merge once at the end in a fixed
-// order.  The visited pairs grow like the mask (O(k) over AR attention)
-// instead of the (N + N k)^2 of a dense mask; dense = 1 visits every key tile
-// with the same per-element mask, the cost of passing the mask densely.
+// A CTA (4 warps) takes 64 consecutive query rows of one (sequence, head),
+// warp w owning rows 16w..16w+15 (FlashAttention-2 layout: no cross-warp
+// merge).  The CTA walks three disjoint key ranges: the context prefix up to
+// the largest context key any of its rows sees, and the block-1 / block-2
+// windows of its rows' groups, in 64-key tiles (cp.async into swizzled shared
+// memory, double-buffered) that all four warps read.  A warp skips a tile
+// none of its rows sees; inside a tile every (row, key) pair is masked by
+// the rule above, except in tiles of context keys every row of the warp sees.
+// S = Q K^T and O += P V run on mma.sync m16n8k16 with P in registers and
+// an online softmax per row.  The visited pairs grow like the mask (O(k) over
+// AR attention) instead of the (N + N k)^2 of a dense mask; dense = 1 visits
+// every key tile with the same per-element mask, the cost of passing the mask
+// densely.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -36,9 +37,9 @@ namespace {
 
 using namespace mma;
 
-constexpr int kTile = 128;     // keys per K/V tile
-constexpr int kThr = 128;
-constexpr int kRows = 16;      // query rows per CTA (the MMA's M)
+constexpr int kTile = 64;      // keys per K/V tile
+constexpr int kThr = 128;      // 4 warps, 16 query rows each
+constexpr int kRows = 64;      // query rows per CTA
 
 struct TrainAttnArgs {
   const __nv_bfloat16* q;      // [B][T][H][64]
@@ -86,41 +87,43 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(128) uint8_t sm[];
-  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(sm);       // [16][64] swizzled
-  __nv_bfloat16* Ks = Qs + kRows * kHD;                           // [2][128][64] swizzled
+  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(sm);       // [64][64] swizzled
+  __nv_bfloat16* Ks = Qs + kRows * kHD;                           // [2][64][64] swizzled
   __nv_bfloat16* Vs = Ks + 2 * kTile * kHD;
 
   const int q0 = a.q_begin + blockIdx.x * kRows, h = blockIdx.y, b = blockIdx.z;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int g = lane >> 2, tq = lane & 3;
   const size_t seq = (size_t)b * a.T;
-  const RowVis v0 = row_vis(a, q0 + g), v1 = row_vis(a, q0 + g + 8);
+  const int qw = q0 + 16 * warp;                                  // this warp's 16 rows
+  const RowVis v0 = row_vis(a, qw + g), v1 = row_vis(a, qw + g + 8);
 
-  // the key ranges of this CTA's rows (every thread computes the same)
+  // key ranges of the CTA's 64 rows (every thread computes the same), and per
+  // warp the context keys all its valid rows see and the last key any sees
   int rlo[3], rhi[3], nr = 0;
-  // context keys every valid row of the tile sees (no mask needed below it)
-  int cmin = 1 << 30;
-  for (int i = 0; i < kRows; ++i) {
-    const RowVis r = row_vis(a, q0 + i);
-    if (r.ctx >= 0) cmin = min(cmin, r.ctx);
-  }
-  if (a.dense) {
-    rlo[0] = 0; rhi[0] = a.T; nr = 1;
-  } else {
+  int wcmin = 1 << 30, wmax = -1;
+  {
     int cmax = -1, w1lo = 1 << 30, w1hi = 0, w2lo = 1 << 30, w2hi = 0;
     for (int i = 0; i < kRows; ++i) {
       const RowVis r = row_vis(a, q0 + i);
       cmax = max(cmax, r.ctx);
       if (r.w1hi > r.w1lo) { w1lo = min(w1lo, r.w1lo); w1hi = max(w1hi, r.w1hi); }
       if (r.w2hi > r.w2lo) { w2lo = min(w2lo, r.w2lo); w2hi = max(w2hi, r.w2hi); }
+      if (i / 16 == warp && r.ctx >= 0) {
+        wcmin = min(wcmin, r.ctx);
+        wmax = max(wmax, max(r.ctx, max(r.w1hi, r.w2hi) - 1));
+      }
     }
-    if (cmax >= 0) { rlo[nr] = 0; rhi[nr] = cmax + 1; ++nr; }
-    if (w1hi > w1lo) { rlo[nr] = w1lo; rhi[nr] = w1hi; ++nr; }
-    if (w2hi > w2lo) { rlo[nr] = w2lo; rhi[nr] = w2hi; ++nr; }
+    if (a.dense) {
+      rlo[0] = 0; rhi[0] = a.T; nr = 1;
+    } else {
+      if (cmax >= 0) { rlo[nr] = 0; rhi[nr] = cmax + 1; ++nr; }
+      if (w1hi > w1lo) { rlo[nr] = w1lo; rhi[nr] = w1hi; ++nr; }
+      if (w2hi > w2lo) { rlo[nr] = w2lo; rhi[nr] = w2hi; ++nr; }
+    }
   }
   int n_tiles = 0;
   for (int i = 0; i < nr; ++i) n_tiles += ceil_div(rhi[i] - rlo[i], kTile);
-  // tile j -> (range, first key)
   auto tile_at = [&](int j, int* lo, int* hi) {
     for (int i = 0; i < nr; ++i) {
       const int n = ceil_div(rhi[i] - rlo[i], kTile);
@@ -147,13 +150,24 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
   };
 
   if (n_tiles > 0) load_tile(0, 0);
-  {
-    // the tile's query rows (zero beyond q_end)
-    const int r = t >> 3, c = t & 7;
+#pragma unroll
+  for (int q = 0; q < kRows * 8 / kThr; ++q) {
+    // the CTA's query rows (zero beyond q_end)
+    const int idx = t + q * kThr;
+    const int r = idx >> 3, c = idx & 7;
     const int qi = q0 + r;
     uint4 val = make_uint4(0, 0, 0, 0);
     if (qi < a.q_end) val = *reinterpret_cast<const uint4*>(a.q + ((seq + qi) * a.H + h) * kHD + c * 8);
     *reinterpret_cast<uint4*>(Qs + swz(r, c)) = val;
+  }
+  __syncthreads();
+  // this warp's Q fragments, kept in registers for every tile
+  uint32_t qa[4][4];
+  {
+    const uint32_t qbase = smem_addr(Qs);
+    const int r = 16 * warp + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks) ldsm_x4(qbase + 2 * swz(r, 2 * ks + (lane >> 4)), qa[ks]);
   }
   // scores in base-2 units: log2(e) / sqrt(hd), applied to S in fp32
   const float sc = 1.4426950408889634f * rsqrtf((float)kHD);
@@ -162,8 +176,6 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
   float o[8][4];
 #pragma unroll
   for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
-  const int kw = warp * 32;
-  const uint32_t qbase = smem_addr(Qs);
 
   for (int it = 0; it < n_tiles; ++it) {
     const int buf = it & 1;
@@ -176,146 +188,102 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
     __syncthreads();
     int kt = 0, kend = 0;
     tile_at(it, &kt, &kend);
-    const uint32_t kbase = smem_addr(Ks + (size_t)buf * kTile * kHD);
-    const uint32_t vbase = smem_addr(Vs + (size_t)buf * kTile * kHD);
-
-    float s[4][4];
+    // warp-uniform: skip a tile none of this warp's rows sees
+    if (kt <= wmax) {
+      const uint32_t kbase = smem_addr(Ks + (size_t)buf * kTile * kHD);
+      const uint32_t vbase = smem_addr(Vs + (size_t)buf * kTile * kHD);
+      // S = Q K^T: 16 rows x 64 keys (n-tile j = keys kt + 8j .. +7)
+      float s[8][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+      for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
 #pragma unroll
-    for (int p = 0; p < 2; ++p) {
-      uint32_t qa0[4], qa1[4];
-      {
-        const int r = (lane & 7) + 8 * ((lane >> 3) & 1);
-        ldsm_x4(qbase + 2 * swz(r, 4 * p + (lane >> 4)), qa0);
-        ldsm_x4(qbase + 2 * swz(r, 4 * p + 2 + (lane >> 4)), qa1);
-      }
+      for (int j = 0; j < 8; ++j) {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        uint32_t kb[4];
-        ldsm_x4(kbase + 2 * swz(kw + 8 * j + (lane & 7), 4 * p + (lane >> 3)), kb);
-        mma16816(s[j], qa0, kb[0], kb[1]);
-        mma16816(s[j], qa1, kb[2], kb[3]);
-      }
-    }
-    // mask: the row's visibility and this tile's range; a warp whose 32
-    // keys are context keys every row sees skips it (rows past q_end have
-    // zero queries and are dropped at the end)
-    const int key0 = kt + kw + 2 * tq;
-    const bool open = kt + kw + 31 < kend && kt + kw + 31 <= cmin && a.dense == 0;
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-    if (open) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          s[j][e] *= sc;
-          s[j][2 + e] *= sc;
-          mx0 = fmaxf(mx0, s[j][e]);
-          mx1 = fmaxf(mx1, s[j][2 + e]);
+        for (int p = 0; p < 2; ++p) {
+          uint32_t kb[4];
+          ldsm_x4(kbase + 2 * swz(8 * j + (lane & 7), 4 * p + (lane >> 3)), kb);
+          mma16816(s[j], qa[2 * p], kb[0], kb[1]);
+          mma16816(s[j], qa[2 * p + 1], kb[2], kb[3]);
         }
       }
-    } else {
+      // mask; a tile of context keys every row of the warp sees needs none
+      const bool open = kt + kTile - 1 < kend && kt + kTile - 1 <= wcmin && a.dense == 0;
+      float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
+      for (int j = 0; j < 8; ++j) {
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
-          const int key = key0 + 8 * j + e;
+          const int key = kt + 8 * j + 2 * tq + e;
           const bool in = key < kend;
-          s[j][e] = (in && sees(v0, key)) ? s[j][e] * sc : -INFINITY;
-          s[j][2 + e] = (in && sees(v1, key)) ? s[j][2 + e] * sc : -INFINITY;
+          s[j][e] = (open || (in && sees(v0, key))) ? s[j][e] * sc : -INFINITY;
+          s[j][2 + e] = (open || (in && sees(v1, key))) ? s[j][2 + e] * sc : -INFINITY;
           mx0 = fmaxf(mx0, s[j][e]);
           mx1 = fmaxf(mx1, s[j][2 + e]);
         }
       }
-    }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float c0 = (mn0 == -INFINITY) ? 1.f : ex2(m0 - mn0);
-    const float c1 = (mn1 == -INFINITY) ? 1.f : ex2(m1 - mn1);
-    m0 = mn0;
-    m1 = mn1;
-    uint32_t pk[4][2];
-    float ps0 = 0.f, ps1 = 0.f;
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float c0 = (mn0 == -INFINITY) ? 1.f : ex2(m0 - mn0);
+      const float c1 = (mn1 == -INFINITY) ? 1.f : ex2(m1 - mn1);
+      m0 = mn0;
+      m1 = mn1;
+      uint32_t pk[8][2];
+      float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      pk[j][0] = (mn0 == -INFINITY) ? 0u : pack_bf16(ex2(s[j][0] - mn0), ex2(s[j][1] - mn0));
-      pk[j][1] = (mn1 == -INFINITY) ? 0u : pack_bf16(ex2(s[j][2] - mn1), ex2(s[j][3] - mn1));
-      const float2 f0 = unpack_bf16(pk[j][0]), f1 = unpack_bf16(pk[j][1]);
-      ps0 += f0.x + f0.y;
-      ps1 += f1.x + f1.y;
-    }
-    l0 = l0 * c0 + ps0;
-    l1 = l1 * c1 + ps1;
+      for (int j = 0; j < 8; ++j) {
+        pk[j][0] = (mn0 == -INFINITY) ? 0u : pack_bf16(ex2(s[j][0] - mn0), ex2(s[j][1] - mn0));
+        pk[j][1] = (mn1 == -INFINITY) ? 0u : pack_bf16(ex2(s[j][2] - mn1), ex2(s[j][3] - mn1));
+        const float2 f0 = unpack_bf16(pk[j][0]), f1 = unpack_bf16(pk[j][1]);
+        ps0 += f0.x + f0.y;
+        ps1 += f1.x + f1.y;
+      }
+      l0 = l0 * c0 + ps0;
+      l1 = l1 * c1 + ps1;
 #pragma unroll
-    for (int nd = 0; nd < 8; ++nd) {
-      o[nd][0] *= c0; o[nd][1] *= c0;
-      o[nd][2] *= c1; o[nd][3] *= c1;
-    }
+      for (int nd = 0; nd < 8; ++nd) {
+        o[nd][0] *= c0; o[nd][1] *= c0;
+        o[nd][2] *= c1; o[nd][3] *= c1;
+      }
+      // O += P V: k-step kk = keys kt + 16kk .. +15
 #pragma unroll
-    for (int kk = 0; kk < 2; ++kk) {
-      const uint32_t pa[4] = {pk[2 * kk][0], pk[2 * kk][1], pk[2 * kk + 1][0], pk[2 * kk + 1][1]};
-      const int vr = kw + 16 * kk + 8 * ((lane >> 3) & 1) + (lane & 7);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint32_t pa[4] = {pk[2 * kk][0], pk[2 * kk][1], pk[2 * kk + 1][0], pk[2 * kk + 1][1]};
+        const int vr = 16 * kk + 8 * ((lane >> 3) & 1) + (lane & 7);
 #pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        uint32_t vb[4];
-        ldsm_x4_t(vbase + 2 * swz(vr, 2 * np + (lane >> 4)), vb);
-        mma16816(o[2 * np], pa, vb[0], vb[1]);
-        mma16816(o[2 * np + 1], pa, vb[2], vb[3]);
+        for (int np = 0; np < 4; ++np) {
+          uint32_t vb[4];
+          ldsm_x4_t(vbase + 2 * swz(vr, 2 * np + (lane >> 4)), vb);
+          mma16816(o[2 * np], pa, vb[0], vb[1]);
+          mma16816(o[2 * np + 1], pa, vb[2], vb[3]);
+        }
       }
     }
     __syncthreads();   // the buffer is refilled next iteration
   }
 
-  // merge the four warps (fixed order)
+  // each warp owns its rows: normalise and store
   l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  float* Ow = reinterpret_cast<float*>(Ks);                     // [4][16][64]
-  float2* ML = reinterpret_cast<float2*>(Ow + 4 * kRows * kHD);  // [4][16]
+  const int qa0 = qw + g, qa1 = qw + g + 8;
+  const size_t nq = (size_t)(a.q_end - a.q_begin);
+  if (qa0 < a.q_end) {
+    const float inv = 1.f / l0;
+    float* dst = a.out + (((size_t)b * nq + (qa0 - a.q_begin)) * a.H + h) * kHD + 2 * tq;
 #pragma unroll
-  for (int nd = 0; nd < 8; ++nd) {
-    *reinterpret_cast<float2*>(Ow + ((size_t)warp * kRows + g) * kHD + 8 * nd + 2 * tq) = make_float2(o[nd][0], o[nd][1]);
-    *reinterpret_cast<float2*>(Ow + ((size_t)warp * kRows + g + 8) * kHD + 8 * nd + 2 * tq) = make_float2(o[nd][2], o[nd][3]);
+    for (int nd = 0; nd < 8; ++nd)
+      *reinterpret_cast<float2*>(dst + 8 * nd) = make_float2(o[nd][0] * inv, o[nd][1] * inv);
   }
-  if (tq == 0) {
-    ML[warp * kRows + g] = make_float2(m0, l0);
-    ML[warp * kRows + g + 8] = make_float2(m1, l1);
-  }
-  __syncthreads();
-  {
-    const int r = t >> 3, d0 = (t & 7) * 8;
-    const int qi = q0 + r;
-    if (qi < a.q_end) {
-      float M = -INFINITY;
+  if (qa1 < a.q_end) {
+    const float inv = 1.f / l1;
+    float* dst = a.out + (((size_t)b * nq + (qa1 - a.q_begin)) * a.H + h) * kHD + 2 * tq;
 #pragma unroll
-      for (int w = 0; w < 4; ++w) M = fmaxf(M, ML[w * kRows + r].x);
-      float wt[4], L = 0.f;
-#pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const float2 ml = ML[w * kRows + r];
-        wt[w] = (ml.x == -INFINITY) ? 0.f : ex2(ml.x - M);
-        L += ml.y * wt[w];
-      }
-      float acc[8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] = 0.f;
-#pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const float4* src = reinterpret_cast<const float4*>(Ow + ((size_t)w * kRows + r) * kHD + d0);
-        const float4 u0 = src[0], u1 = src[1];
-        acc[0] += u0.x * wt[w]; acc[1] += u0.y * wt[w]; acc[2] += u0.z * wt[w]; acc[3] += u0.w * wt[w];
-        acc[4] += u1.x * wt[w]; acc[5] += u1.y * wt[w]; acc[6] += u1.z * wt[w]; acc[7] += u1.w * wt[w];
-      }
-      const float inv = 1.f / L;
-      float* dst = a.out + (((size_t)b * (a.q_end - a.q_begin) + (qi - a.q_begin)) * a.H + h) * kHD + d0;
-      *reinterpret_cast<float4*>(dst) = make_float4(acc[0] * inv, acc[1] * inv, acc[2] * inv, acc[3] * inv);
-      *reinterpret_cast<float4*>(dst + 4) = make_float4(acc[4] * inv, acc[5] * inv, acc[6] * inv, acc[7] * inv);
-    }
+    for (int nd = 0; nd < 8; ++nd)
+      *reinterpret_cast<float2*>(dst + 8 * nd) = make_float2(o[nd][2] * inv, o[nd][3] * inv);
   }
 }
 
