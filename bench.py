@@ -220,6 +220,17 @@ def cpu_threads():
 
 
 # ------------------------------------------------------------------ main
+def bench_config(w, B, gen, k):
+    """The `config` object of the bench line (both arms)."""
+    model = w.model
+    return {"workload": f"{w.name}: {model.n_layer}L d{model.d_model} H{model.n_head} "
+                        f"F{model.d_ff} V{model.vocab}, batch {B}, prompt "
+                        f"{w.prompt_len or 'ragged'} +{gen} tokens, k={k}",
+            "batch": B, "k": k, "gen_tokens_per_seq": gen,
+            "calls_per_step": -(-gen // max(k, 1)), "map": model.map,
+            "l2": "working set larger than L2 (weights + KV), no flush"}
+
+
 def workload_of(args):
     from synth import WORKLOADS
     w = WORKLOADS[args.workload]
@@ -253,7 +264,7 @@ def run_reference(args):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000 * el / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": f"{w.name}: batch {B}, k={args.k}", "batch": B, "k": args.k},
+            "config": bench_config(w, B, gen, args.k),
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cpu_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -674,12 +685,7 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": model.dtype, "data": "synthetic: seeded N(0,0.02) weights, uniform prompt ids, U[0,1) noise",
-            "config": {"workload": f"{w.name}: {model.n_layer}L d{model.d_model} H{model.n_head} "
-                                   f"F{model.d_ff} V{model.vocab}, batch {B}, prompt "
-                                   f"{w.prompt_len or 'ragged'} +{gen} tokens, k={k}",
-                       "batch": B, "k": k, "gen_tokens_per_seq": gen,
-                       "calls_per_step": calls, "map": model.map,
-                       "l2": "working set larger than L2 (weights + KV), no flush"},
+            "config": bench_config(w, B, gen, k),
             "k1": ar,
             "speedup_k_vs_k1": (val / ar["value"]) if ar else None,
             "step_roofline_frac": step_frac,
