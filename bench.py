@@ -619,7 +619,7 @@ def main():
         ar_val, ar_ms, ar_calls, _ = measure(0)
         ar = {"value": ar_val, "unit": "tokens/s", "ms_per_step": ar_ms, "calls_per_step": ar_calls}
 
-    # per-kernel times over one eager step near the middle of the generation
+    # per-kernel times over one profiled step (a graph with event nodes) near the middle of the generation
     dec.rewind()
     zmid = np.random.default_rng(5).random((B, nout), dtype=np.float32)
     out = np.zeros((B, nout), np.int32)

@@ -219,8 +219,9 @@ int kf_set_stream(kf_ctx* ctx, void* stream);
 int kf_sync(kf_ctx* ctx);
 
 /*
- * Profiling aid: run one decode step like kf_decode_step but eagerly, with a
- * CUDA event pair around every launch.  ms_per_kind[i] and launches_per_kind[i]
+ * Profiling aid: run one decode step like kf_decode_step, as a one-off CUDA
+ * graph with an event record node on each side of every launch (launches in
+ * order, without programmatic dependent launch).  ms_per_kind[i] and launches_per_kind[i]
  * (arrays of KF_KIND_COUNT, host) receive the summed device time and launch
  * count per kernel kind.  Synchronises.
  */

@@ -168,13 +168,14 @@ struct PdlScope {
 static void prof_begin(kf_ctx* c, int kind) {
   if (!c->prof) return;
   if (c->ev_used + 2 > (int)c->ev.size()) return;
-  cudaEventRecord(c->ev[c->ev_used], c->stream);
+  // recorded while the profiled step is captured: an event record node
+  cudaEventRecordWithFlags(c->ev[c->ev_used], c->stream, cudaEventRecordExternal);
   c->ev_kind[c->ev_used / 2] = kind;
 }
 static void prof_end(kf_ctx* c) {
   if (!c->prof) return;
   if (c->ev_used + 2 > (int)c->ev.size()) return;
-  cudaEventRecord(c->ev[c->ev_used + 1], c->stream);
+  cudaEventRecordWithFlags(c->ev[c->ev_used + 1], c->stream, cudaEventRecordExternal);
   c->ev_used += 2;
 }
 
@@ -903,10 +904,30 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
         c->ev_kind.resize(2048);
         for (auto& ev : c->ev) KF_CUDA(cudaEventCreate(&ev));
       }
+      // the profiled step replays as a graph with the event records as nodes,
+      // so each event pair brackets its kernel and not the host's launch work
+      cudaGraph_t g = nullptr;
+      cudaGraphExec_t exec = nullptr;
+      KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
+      enqueue_step(c, B, P, k, c->noise);
+      c->prof = false;
+      cudaError_t e1 = cudaGetLastError();
+      cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
+      if (e1 != cudaSuccess && g) cudaGraphDestroy(g);
+      if (e1 != cudaSuccess) return cuda_fail(c, e1, "profile capture");
+      if (e2 != cudaSuccess) return cuda_fail(c, e2, "profile cudaStreamEndCapture");
+      cudaError_t e3 = cudaGraphInstantiate(&exec, g, 0);
+      cudaGraphDestroy(g);
+      if (e3 != cudaSuccess) return cuda_fail(c, e3, "profile cudaGraphInstantiate");
+      cudaError_t e4 = cudaGraphLaunch(exec, c->stream);
+      cudaError_t e5 = cudaStreamSynchronize(c->stream);
+      cudaGraphExecDestroy(exec);
+      if (e4 != cudaSuccess) return cuda_fail(c, e4, "profile cudaGraphLaunch");
+      if (e5 != cudaSuccess) return cuda_fail(c, e5, "profile step");
+    } else {
+      enqueue_step(c, B, P, k, c->noise);
+      KF_CUDA(cudaGetLastError());
     }
-    enqueue_step(c, B, P, k, c->noise);
-    c->prof = false;
-    KF_CUDA(cudaGetLastError());
   }
   KF_CUDA(cudaMemcpyAsync(out_tokens, c->tokens, (size_t)B * nout * 4, cudaMemcpyDefault, c->stream));
   for (int b = 0; b < B; ++b) c->h_len[b] += P;

@@ -159,6 +159,30 @@ def test_pdl_equals_plain_launches(kf):
             np.testing.assert_array_equal(a, b)
 
 
+def test_profile_step_matches_decode(kf, lm1b_weights):
+    """kf_profile_step (a one-off graph with event nodes) decodes exactly like
+    kf_decode_step and reports every launch of the step."""
+    cfg = LM1B
+    prompts = make_prompts([20, 33], cfg.vocab)
+    a = kf.Decoder(cfg, lm1b_weights, max_batch=2, max_k=4)
+    b = kf.Decoder(cfg, lm1b_weights, max_batch=2, max_k=4)
+    a.prefill(prompts)
+    b.prefill(prompts)
+    rng = np.random.default_rng(12)
+    for k in (4, 4, 0):
+        z = rng.random((2, max(k, 1)), dtype=np.float32)
+        ta = np.zeros((2, max(k, 1)), np.int32)
+        ms = np.zeros(kf.KF_KIND_COUNT, np.float32)
+        n = np.zeros(kf.KF_KIND_COUNT, np.int32)
+        kf.kf_profile_step(a.ctx, 2, k, z, ta, ms, n)
+        assert np.array_equal(ta, b.step(k, z))
+        names = dict(zip(kf.KIND_NAMES, zip(ms, n)))
+        assert names["gemm_qkv"][1] == cfg.n_layer and names["attention"][1] == cfg.n_layer
+        assert all(t > 0 for t, c in names.values() if c > 0)
+    a.close()
+    b.close()
+
+
 def test_norm_gains_folded(kf):
     """Non-unit RMSNorm gains: the fused path folds them into the QKV and
     MLP-up weights; the oracle applies them after normalising."""
