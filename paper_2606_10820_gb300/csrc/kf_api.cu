@@ -95,6 +95,7 @@ struct kf_ctx {
   std::map<std::tuple<int, int, int>, cudaGraphExec_t> graphs;
   // profiling
   bool prof = false;
+  bool launch_failed = false;   // a launch refused on the host (e.g. a TMA descriptor)
   std::vector<cudaEvent_t> ev;
   std::vector<int> ev_kind;
   int ev_used = 0;
@@ -123,6 +124,15 @@ static int cuda_fail(kf_ctx* c, cudaError_t e, const char* what) {
     cudaError_t e_ = (call);                                \
     if (e_ != cudaSuccess) return cuda_fail(c, e_, #call);  \
   } while (0)
+
+// status of the launches enqueued since the last call: a CUDA error, or a
+// launch the host refused to make
+static cudaError_t enqueue_status(kf_ctx* c) {
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && c->launch_failed) e = cudaErrorInvalidValue;
+  c->launch_failed = false;
+  return e;
+}
 
 static bool is_device_ptr(const void* p) {
   cudaPointerAttributes at;
@@ -185,8 +195,9 @@ static void gemm(kf_ctx* c, int kind, int M, int N, int K, const void* A, int ld
   GemmDesc g{M, N, K, A, lda, W, ldw, e};
   prof_begin(c, kind);
   bool use_tc = c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && tc_gemm_supported(g);
-  if (use_tc)
-    launch_gemm_tc(g, c->d_err, c->stream);
+  if (use_tc) {
+    if (launch_gemm_tc(g, c->d_err, c->stream) != 0) c->launch_failed = true;
+  }
   else
     launch_gemm_simt(c->bf16, g, c->stream);
   prof_end(c);
@@ -264,7 +275,9 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.len = groups ? nullptr : c->d_len;   // decode: keys below it are stable during the step
     prof_begin(c, KF_KIND_ATTENTION);
     if (tc_attn) launch_attention_tc(a, n_groups, s);
-    else if (mma_attn) launch_attention_mma(a, n_groups, c->cfg.max_len, s);
+    else if (mma_attn) {
+      if (launch_attention_mma(a, n_groups, rows, c->cfg.max_len, s) != 0) c->launch_failed = true;
+    }
     else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
     if (n_split > 1) {
@@ -632,7 +645,7 @@ static int prefill_rows(kf_ctx* c, const std::vector<PrefillSeq>& seqs) {
                           c->stream);
       enqueue_layers(c, R, (int)grp.size(), c->groups, 0);
     }
-    KF_CUDA(cudaGetLastError());
+    KF_CUDA(enqueue_status(c));
     // the host vectors are reused: wait until the copies have consumed them
     KF_CUDA(cudaStreamSynchronize(c->stream));
     r_tok.clear(); r_seq.clear(); r_pos.clear(); grp.clear();
@@ -825,7 +838,7 @@ int kf_teacher_step(kf_ctx* c, int32_t B, int32_t k, const float* noise, int32_t
       cudaGraph_t g = nullptr;
       KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
       enqueue();
-      cudaError_t e1 = cudaGetLastError();
+      cudaError_t e1 = enqueue_status(c);
       cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
       if (e1 != cudaSuccess) return cuda_fail(c, e1, "capture launch");
       if (e2 != cudaSuccess) return cuda_fail(c, e2, "cudaStreamEndCapture");
@@ -839,7 +852,7 @@ int kf_teacher_step(kf_ctx* c, int32_t B, int32_t k, const float* noise, int32_t
     KF_CUDA(cudaGraphLaunch(exec, c->stream));
   } else {
     enqueue();
-    KF_CUDA(cudaGetLastError());
+    KF_CUDA(enqueue_status(c));
   }
   KF_CUDA(cudaMemcpyAsync(out_tokens, c->t_out, (size_t)B * k * 4, cudaMemcpyDefault, c->stream));
   for (int b = 0; b < B; ++b) c->h_len[b] += P + k - 1;
@@ -883,7 +896,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
       cudaGraph_t g = nullptr;
       KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
       enqueue_step(c, B, P, k, c->noise);
-      cudaError_t e1 = cudaGetLastError();
+      cudaError_t e1 = enqueue_status(c);
       cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
       if (e1 != cudaSuccess) return cuda_fail(c, e1, "capture launch");
       if (e2 != cudaSuccess) return cuda_fail(c, e2, "cudaStreamEndCapture");
@@ -911,7 +924,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
       KF_CUDA(cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal));
       enqueue_step(c, B, P, k, c->noise);
       c->prof = false;
-      cudaError_t e1 = cudaGetLastError();
+      cudaError_t e1 = enqueue_status(c);
       cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
       if (e1 != cudaSuccess && g) cudaGraphDestroy(g);
       if (e1 != cudaSuccess) return cuda_fail(c, e1, "profile capture");
@@ -926,7 +939,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
       if (e5 != cudaSuccess) return cuda_fail(c, e5, "profile step");
     } else {
       enqueue_step(c, B, P, k, c->noise);
-      KF_CUDA(cudaGetLastError());
+      KF_CUDA(enqueue_status(c));
     }
   }
   KF_CUDA(cudaMemcpyAsync(out_tokens, c->tokens, (size_t)B * nout * 4, cudaMemcpyDefault, c->stream));
@@ -993,7 +1006,7 @@ int kf_debug_logits(kf_ctx* c, float* out) {
     e.kind = EPI_LOGITS; e.outf = dst; e.ldo = c->V; e.inv_tau = 1.0f / c->cfg.tau; e.n_valid = c->V;
     gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, c->d, c->head_in, c->d, c->w_head, c->d, e);
   }
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = enqueue_status(c);
   if (err == cudaSuccess && !dev)
     err = cudaMemcpyAsync(out, tmp, (size_t)nh * c->V * 4, cudaMemcpyDeviceToHost, c->stream);
   if (err == cudaSuccess) err = cudaStreamSynchronize(c->stream);

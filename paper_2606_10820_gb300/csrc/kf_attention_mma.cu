@@ -4,16 +4,20 @@
 // at or before each row's position (the fully causal mask of Sec. 3.3 /
 // Alg. 1).
 //
-// Per CTA (4 warps), keys in tiles of 128 streamed into shared memory with
-// 16-byte cp.async (double-buffered when the CTA sees more than one tile);
-// rows are XOR-swizzled in 16-byte chunks so ldmatrix reads are
-// conflict-free without padding.  Warp w owns keys 32w .. 32w+31 of every
-// tile and keeps its own online softmax over them (FlashAttention-2 style):
+// Per CTA (4 warps), keys in tiles of 128 (8 pages).  Each page of K and of
+// V for the CTA's head is 16 contiguous 128-byte rows of the cache; one TMA
+// copy per page and operand lands it 128-byte swizzled (16-byte chunk c of
+// row r at chunk c ^ (r % 8)), so ldmatrix reads are conflict-free, and one
+// mbarrier per buffer counts the bytes.  NBUF = 2: a ring of two buffers,
+// the next tile in flight while one is reduced.  Warp w owns keys
+// 32w .. 32w+31 of every tile and keeps its own online softmax over them
+// (FlashAttention-2 style):
 //   S = Q K^T      16 rows x 32 keys, 16 MMAs (Q zero-padded to 16 rows)
 //   P = exp(S - m) in registers; the S accumulator layout is the A-operand
 //                  layout of the next MMA, so P never leaves the registers
 //   O += P V       16 rows x 64 dims, 16 MMAs (V through ldmatrix.trans)
-// The four warps' (m, l, O) are merged once at the end in a fixed order
+// Only tiles that reach past the first row's position are masked.  The four
+// warps' (m, l, O) are merged once at the end in a fixed order
 // (deterministic); with n_split > 1 each CTA covers one key range and
 // k_attn_combine merges the partial softmaxes in split order.
 //
@@ -26,8 +30,8 @@
 
 #include <algorithm>
 
-#include "kf_internal.cuh"
 #include "kf_mma.cuh"
+#include "kf_tc.cuh"
 
 namespace kf {
 namespace {
@@ -37,31 +41,38 @@ using namespace mma;
 constexpr int kTile = 128;     // keys per K/V tile
 constexpr int kThr = 128;      // 4 warps x 32 keys of each tile
 constexpr int kQRows = 16;     // MMA M: query rows of the group, zero-padded
+constexpr int kPageBytes = kPage * kHD * 2;                  // one page of K (or V) of one head
+constexpr int kTileBytes = kTile * kHD * 2;                  // 16 KB
 
-constexpr size_t smem_bytes(int nbuf) {
-  return (size_t)kQRows * kHD * 2 + (size_t)nbuf * 2 * kTile * kHD * 2;
+// [NBUF K tiles][NBUF V tiles][Q 16 x 64][NBUF mbarriers][page ids], from a
+// 1024-byte aligned base (the swizzle pattern repeats every 8 rows)
+constexpr size_t smem_bytes(int nbuf, int pg_cap) {
+  return 1024 + (size_t)2 * nbuf * kTileBytes + (size_t)kQRows * kHD * 2 + 8 * nbuf + 4 * pg_cap;
 }
 
 }  // namespace
 
-// NBUF = 1: CTAs of at most one key tile; NBUF = 2: double-buffered tiles.
-// Single-tile decode CTAs (a.len set, one group per sequence): the keys before the
+// NBUF = 1: CTAs of at most one key tile; NBUF = 2: two tile buffers.  TWO:
+// groups of more than 8 rows (rows 8..15 of the MMA carry data).  Decode
+// CTAs (a.len set, one group per sequence): the pages wholly before the
 // sequence's committed length were written by earlier steps and the page
-// table by the host before the step, so the copies of those keys are issued
-// before waiting for the kernel that appends this step's keys; the new keys
-// and Q are loaded after the wait.
-template <int NBUF>
-__global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnArgs a) {
+// table by the host before the step, so the page ids and the copies of those
+// pages are issued before waiting for the kernel that appends this step's
+// keys; the other pages and Q are loaded after the wait.
+template <int NBUF, bool TWO>
+__global__ void __launch_bounds__(kThr, NBUF == 1 ? (TWO ? 5 : 6) : 3)
+k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
   pdl_trigger();
-  extern __shared__ __align__(128) uint8_t sm[];
-  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(sm);   // [16][64] swizzled
-  __nv_bfloat16* Ks = Qs + kQRows * kHD;                      // [NBUF][128][64] swizzled
+  extern __shared__ __align__(1024) uint8_t sm_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
+  __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(sm);   // [NBUF][128][64] swizzled
   __nv_bfloat16* Vs = Ks + NBUF * kTile * kHD;                // [NBUF][128][64] swizzled
+  __nv_bfloat16* Qs = Vs + NBUF * kTile * kHD;                // [16][64] swizzled
+  uint64_t* bars = reinterpret_cast<uint64_t*>(Qs + kQRows * kHD);
+  int* s_pg = reinterpret_cast<int*>(bars + NBUF);            // [a.pg_cap] (NBUF = 2)
 
   const int gi = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
-  // (single-tile CTAs only: with several tiles the double buffer hides the
-  // first tile's latency already)
-  const bool early = NBUF == 1 && a.len != nullptr && a.groups == nullptr;
+  const bool early = a.len != nullptr && a.groups == nullptr;
   int b, row0, nr, n_keys, stable;
   if (early) {
     b = gi; row0 = gi * a.uniform_rows; nr = a.uniform_rows;
@@ -83,66 +94,87 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int g = lane >> 2, tq = lane & 3;     // MMA fragment row group / column pair
 
-  const __nv_bfloat16* kv = reinterpret_cast<const __nv_bfloat16*>(a.kv);
-  const size_t head_page = (size_t)kPage * kHD;
-  const size_t layer_base = (size_t)a.layer * a.n_pages * 2 * a.H * head_page;
-  bool bad_page = false;
-
-  // cp.async of the keys [key_lo, key_hi) of the tile starting at kt into
-  // buffer buf (keys >= k_end are zero-filled).  kt is a multiple of the page
-  // size: thread t copies chunk t % 8 of keys kt + t / 8 + 16 q, i.e. one key
-  // of page kt / 16 + q for q = 0..7; the page ids are all fetched before the
-  // first copy is issued.
-  auto load_tile = [&](int kt, int buf, int key_lo, int key_hi) {
-    __nv_bfloat16* kd = Ks + (size_t)buf * kTile * kHD;
-    __nv_bfloat16* vd = Vs + (size_t)buf * kTile * kHD;
-    constexpr int NQ = kTile * 8 / kThr;
-    static_assert(kThr / 8 == kPage, "one page per copy round");
-    int pg[NQ];
-#pragma unroll
-    for (int q = 0; q < NQ; ++q) {
-      const int pi = kt / kPage + q;
-      const int kq = kt + q * kPage;        // first key of the page
-      pg[q] = (kq < k_end && kq + kPage > key_lo && kq < key_hi && pi < a.max_pages)
-                  ? __ldg(a.page_table + b * a.max_pages + pi) : -1;
-    }
-#pragma unroll
-    for (int q = 0; q < NQ; ++q) {
-      const int idx = t + q * kThr;
-      const int j = idx >> 3, c = idx & 7;
-      const int key = kt + j;
-      if (key < key_lo || key >= key_hi) continue;
-      const __nv_bfloat16* src = kv;
-      int nbytes = 0;
-      if (key < k_end) {
-        const int page = pg[q];
-        if (page >= 0 && page < a.n_pages) {
-          src = kv + layer_base + (((size_t)page * 2) * a.H + h) * head_page + (size_t)(key % kPage) * kHD + c * 8;
-          nbytes = 16;
-        } else {
-          bad_page = true;
-        }
-      }
-      cp_async16(smem_addr(kd + swz(j, c)), src, nbytes);
-      cp_async16(smem_addr(vd + swz(j, c)), src + (nbytes ? a.H * head_page : 0), nbytes);
-    }
-    cp_commit();
-  };
-
   int n_tiles = k_end > k_begin ? ceil_div(k_end - k_begin, kTile) : 0;
   if (NBUF == 1 && n_tiles > 1) {
     // the single-buffer variant is launched only for CTAs of at most one tile
     if (t == 0) atomicOr(a.d_err, kErrInternal);
     n_tiles = 1;
   }
-  if (n_tiles > 0) {
-    // first tile: its stable keys now, the rest after the wait
-    const int split_key = early ? max(k_begin, min(stable, k_begin + kTile)) : k_begin;
-    if (split_key > k_begin) load_tile(k_begin, 0, k_begin, split_key);
-    if (early) pdl_wait();
-    load_tile(k_begin, 0, split_key, k_begin + kTile);
-  } else if (early) {
-    pdl_wait();
+  const int pg0 = k_begin / kPage;            // k_begin is a multiple of the page size
+  int n_pg = 0;
+  if constexpr (NBUF > 1) {
+    // the page ids of the keys [k_begin, k_end)
+    n_pg = k_end > k_begin ? ceil_div(k_end, kPage) - pg0 : 0;
+    if (n_pg > a.pg_cap) {
+      if (t == 0) atomicOr(a.d_err, kErrInternal);
+      n_pg = a.pg_cap;
+    }
+    for (int i = t; i < n_pg; i += kThr)
+      s_pg[i] = pg0 + i < a.max_pages ? __ldg(a.page_table + (size_t)b * a.max_pages + pg0 + i) : -1;
+  }
+  // V rows of pages that are not copied (past the last key) stay finite: the
+  // masked keys' probabilities are 0 and 0 * V must be 0
+  for (int i = t; i < NBUF * kTile * kHD / 8; i += kThr)
+    reinterpret_cast<uint4*>(Vs)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (t == 0) {
+    for (int i = 0; i < NBUF; ++i) mbar_init(smem_u32(&bars[i]), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // zeros before the copies
+  __syncthreads();
+
+  // Copies of the pages of the tile at kt whose first key lies in
+  // [key_lo, key_hi) (multiples of the page size) into buffer buf, by lanes
+  // 0..7 of warp 0 (one page each).  The bytes are added to the buffer's
+  // mbarrier; `arrive` completes its single arrival (the last part of a tile).
+  auto issue = [&](int kt, int buf, int key_lo, int key_hi, bool arrive) {
+    if (warp != 0) return;
+    const int kq = kt + lane * kPage;         // first key of this lane's page
+    int page = -1;
+    bool go = false;
+    if (lane < kTile / kPage && kq < k_end && kq >= key_lo && kq < key_hi) {
+      const int pi = kq / kPage;
+      if constexpr (NBUF == 1)
+        page = pi < a.max_pages ? __ldg(a.page_table + (size_t)b * a.max_pages + pi) : -1;
+      else
+        page = pi - pg0 < n_pg ? s_pg[pi - pg0] : -1;
+      go = page >= 0 && page < a.n_pages;
+      if (!go) atomicOr(a.d_err, kErrBadPage);
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, go);
+    const uint32_t bar = smem_u32(&bars[buf]);
+    if (lane == 0) {
+      const uint32_t bytes = (uint32_t)__popc(m) * 2u * kPageBytes;
+      if (arrive)
+        mbar_expect_tx(bar, bytes);
+      else if (bytes)
+        asm volatile("mbarrier.expect_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+    }
+    __syncwarp();
+    if (go) {
+      const int row = (page * 2 * a.H + h) * kPage;   // K rows; V rows follow H pages later
+      const uint32_t off = (uint32_t)(buf * kTileBytes + lane * kPageBytes);
+      tma_load_2d(smem_u32(Ks) + off, &map_kv, bar, 0, row);
+      tma_load_2d(smem_u32(Vs) + off, &map_kv, bar, 0, row + a.H * kPage);
+    }
+  };
+
+  // the first tiles: pages wholly below the committed length now, the rest
+  // after the wait
+  {
+    const int pre = min(NBUF, n_tiles);
+    const int cut = early ? (stable / kPage) * kPage : k_begin;   // first page not yet stable
+    if (early) {
+      for (int i = 0; i < pre; ++i) {
+        const int kt = k_begin + i * kTile;
+        issue(kt, i, kt, min(cut, kt + kTile), false);
+      }
+      pdl_wait();
+    }
+    for (int i = 0; i < pre; ++i) {
+      const int kt = k_begin + i * kTile;
+      issue(kt, i, max(kt, cut), kt + kTile, true);
+    }
   }
   const int pos0 = g < nr ? a.row_pos[row0 + g] : -1;          // rows g and g + 8
   const int pos1 = g + 8 < nr ? a.row_pos[row0 + g + 8] : -1;
@@ -171,19 +203,15 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
 #pragma unroll
   for (int nd = 0; nd < 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
   const int kw = warp * 32;               // this warp's keys within a tile
-  const bool two = nr > 8;                // rows 8..15 exist (else zero padding)
   const uint32_t qbase = smem_addr(Qs);
+  // keys every row of the group sees: those at or before the first row's position
+  const int full_end = min(k_end, nr > 0 ? a.row_pos[row0] + 1 : 0);
+  __syncthreads();                        // Q
 
   for (int it = 0; it < n_tiles; ++it) {
     const int kt = k_begin + it * kTile;
-    const int buf = (NBUF == 2) ? (it & 1) : 0;
-    if (NBUF == 2 && it + 1 < n_tiles) {
-      load_tile(kt + kTile, buf ^ 1, kt + kTile, kt + 2 * kTile);
-      cp_wait<1>();
-    } else {
-      cp_wait<0>();
-    }
-    __syncthreads();
+    const int buf = it % NBUF;
+    mbar_wait(smem_u32(&bars[buf]), (uint32_t)(it / NBUF) & 1u, a.d_err);
     const uint32_t kbase = smem_addr(Ks + (size_t)buf * kTile * kHD);
     const uint32_t vbase = smem_addr(Vs + (size_t)buf * kTile * kHD);
 
@@ -208,29 +236,35 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
       }
     }
 
-    // causal mask and online softmax (per warp)
-    const int key0 = kt + kw + 2 * tq;
+    // causal mask (tiles past the first row's position only) and online
+    // softmax (per warp)
+    if (kt + kTile > full_end) {
+      const int key0 = kt + kw + 2 * tq;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = key0 + 8 * j + e;
+          if (!(key < k_end && key <= pos0)) s[j][e] = -INFINITY;
+          if (TWO && !(key < k_end && key <= pos1)) s[j][2 + e] = -INFINITY;
+        }
+      }
+    }
     float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int key = key0 + 8 * j + e;
-        if (!(key < k_end && key <= pos0)) s[j][e] = -INFINITY;
-        if (!(key < k_end && key <= pos1)) s[j][2 + e] = -INFINITY;
-        mx0 = fmaxf(mx0, s[j][e]);
-        mx1 = fmaxf(mx1, s[j][2 + e]);
-      }
+      mx0 = fmaxf(mx0, fmaxf(s[j][0], s[j][1]));
+      if (TWO) mx1 = fmaxf(mx1, fmaxf(s[j][2], s[j][3]));
     }
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    if (two) {
+    if (TWO) {
       mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
       mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
     }
     const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
     const float c0 = (mn0 == -INFINITY) ? 1.f : ex2(m0 - mn0);
-    const float c1 = (mn1 == -INFINITY) ? 1.f : ex2(m1 - mn1);
+    const float c1 = (!TWO || mn1 == -INFINITY) ? 1.f : ex2(m1 - mn1);
     m0 = mn0;
     m1 = mn1;
     // probabilities as bf16 pairs (the MMA A operand); the sums use the
@@ -243,7 +277,7 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
       const float2 f0 = unpack_bf16(pk[j][0]);
       ps0 += f0.x + f0.y;
       pk[j][1] = 0u;
-      if (two) {
+      if (TWO) {
         pk[j][1] = (mn1 == -INFINITY) ? 0u : pack_bf16(ex2(s[j][2] - mn1), ex2(s[j][3] - mn1));
         const float2 f1 = unpack_bf16(pk[j][1]);
         ps1 += f1.x + f1.y;
@@ -254,7 +288,7 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
 #pragma unroll
     for (int nd = 0; nd < 8; ++nd) {
       o[nd][0] *= c0; o[nd][1] *= c0;
-      o[nd][2] *= c1; o[nd][3] *= c1;
+      if (TWO) { o[nd][2] *= c1; o[nd][3] *= c1; }
     }
 
     // O += P V: k-step kk = keys kw + 16kk .. +15; V fragments by ldmatrix.trans
@@ -270,9 +304,12 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
         mma16816(o[2 * np + 1], pa, vb[2], vb[3]);
       }
     }
-    __syncthreads();   // the buffer is refilled next iteration
+    __syncthreads();   // buffer buf is free: tile it + NBUF goes there
+    if (it + NBUF < n_tiles) {
+      const int kn = kt + NBUF * kTile;
+      issue(kn, buf, kn, kn + kTile, true);
+    }
   }
-  if (bad_page) atomicOr(a.d_err, kErrBadPage);
 
   // merge the four warps (fixed order): per warp m, l and O of the 16 rows
   l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
@@ -338,24 +375,39 @@ __global__ void __launch_bounds__(kThr, NBUF == 1 ? 6 : 3) k_attention_mma(AttnA
   }
 }
 
-template <int NBUF>
-static void launch_nb(const AttnArgs& a, int n_groups, cudaStream_t s) {
-  const size_t smem = smem_bytes(NBUF);
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(k_attention_mma<NBUF>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    attr = true;
+template <int NBUF, bool TWO>
+static void launch_nb(const CUtensorMap& map, const AttnArgs& a, int n_groups, cudaStream_t s) {
+  static size_t attr = 0;
+  const size_t smem = smem_bytes(NBUF, a.pg_cap);
+  if (smem > attr) {
+    cudaFuncSetAttribute(k_attention_mma<NBUF, TWO>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    attr = smem;
   }
-  kf_launch(k_attention_mma<NBUF>, dim3(n_groups, a.H, a.n_split), dim3(kThr), smem, s, a);
+  kf_launch(k_attention_mma<NBUF, TWO>, dim3(n_groups, a.H, a.n_split), dim3(kThr), smem, s, map, a);
 }
 
 bool attention_mma_supported(bool bf16, int hd, int rows) { return bf16 && hd == kHD && rows <= kQRows; }
 
-void launch_attention_mma(const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s) {
-  if (n_groups == 0) return;
-  // one K/V buffer when no CTA sees more than one tile of keys
-  if (std::min(a.keys_per_split, max_keys) <= kTile) launch_nb<1>(a, n_groups, s);
-  else launch_nb<2>(a, n_groups, s);
+int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_keys, cudaStream_t s) {
+  if (n_groups == 0) return 0;
+  AttnArgs a = a0;
+  const int keys = std::min(a.keys_per_split, max_keys);   // the most keys of one CTA
+  a.pg_cap = ceil_div(keys, kPage);
+  // this layer's K/V pages as rows of 64 bf16: ((page * 2 + kv) * H + head) * 16 + key
+  const size_t layer_elems = (size_t)a.n_pages * 2 * a.H * kPage * kHD;
+  CUtensorMap map;
+  if (!encode_rows_map_bf16(&map, static_cast<const __nv_bfloat16*>(a.kv) + (size_t)a.layer * layer_elems,
+                            (uint64_t)a.n_pages * 2 * a.H * kPage, kHD, kPage))
+    return -1;
+  const bool two = rows > 8;
+  if (keys <= kTile) {
+    if (two) launch_nb<1, true>(map, a, n_groups, s);
+    else launch_nb<1, false>(map, a, n_groups, s);
+  } else {
+    if (two) launch_nb<2, true>(map, a, n_groups, s);
+    else launch_nb<2, false>(map, a, n_groups, s);
+  }
+  return 0;
 }
 
 }  // namespace kf

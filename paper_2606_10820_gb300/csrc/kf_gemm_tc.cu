@@ -440,6 +440,17 @@ static bool make_map(CUtensorMap* m, const void* ptr, int rows, int cols, int ld
   return r == CUDA_SUCCESS;
 }
 
+bool encode_rows_map_bf16(CUtensorMap* m, const void* base, uint64_t rows, int cols, int box_rows) {
+  if (!get_encode() || (reinterpret_cast<uintptr_t>(base) & 15) || (cols * 2) % 16) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {(cuuint32_t)cols, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool tc_gemm_supported(const GemmDesc& g) {
   if (g.K % kBK || g.K == 0 || g.M <= 0 || g.N <= 0) return false;
   if ((g.lda * 2) % 16 || (g.ldw * 2) % 16) return false;
@@ -531,16 +542,16 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
   return cudaLaunchKernelEx(&cfg, k_gemm_tc<BN, STAGES, EPI, MT, AT>, ma, mw, a) == cudaSuccess ? 0 : -1;
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int AT>
 static int launch_bn(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s) {
   switch (g.epi.kind) {
-    case EPI_STORE: return launch_epi<BN, STAGES, EPI_STORE>(g, d_err, num_sms, s);
-    case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU>(g, d_err, num_sms, s);
-    case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID>(g, d_err, num_sms, s);
-    case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT>(g, d_err, num_sms, s);
-    case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS>(g, d_err, num_sms, s);
-    case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32>(g, d_err, num_sms, s);
-    case EPI_QKV: return launch_epi<BN, STAGES, EPI_QKV>(g, d_err, num_sms, s);
+    case EPI_STORE: return launch_epi<BN, STAGES, EPI_STORE, 1, AT>(g, d_err, num_sms, s);
+    case EPI_BIAS_GELU: return launch_epi<BN, STAGES, EPI_BIAS_GELU, 1, AT>(g, d_err, num_sms, s);
+    case EPI_RESID: return launch_epi<BN, STAGES, EPI_RESID, 1, AT>(g, d_err, num_sms, s);
+    case EPI_NOISE_OUT: return launch_epi<BN, STAGES, EPI_NOISE_OUT, 1, AT>(g, d_err, num_sms, s);
+    case EPI_LOGITS: return launch_epi<BN, STAGES, EPI_LOGITS, 1, AT>(g, d_err, num_sms, s);
+    case EPI_STORE_F32: return launch_epi<BN, STAGES, EPI_STORE_F32, 1, AT>(g, d_err, num_sms, s);
+    case EPI_QKV: return launch_epi<BN, STAGES, EPI_QKV, 1, AT>(g, d_err, num_sms, s);
   }
   return -1;
 }
@@ -558,11 +569,14 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
     if (g.M > kBM) return launch_epi<256, 3, EPI_HEAD, 2, 1>(g, d_err, num_sms, s);
     return launch_epi<256, 2, EPI_HEAD, 1, 2>(g, d_err, num_sms, s);
   }
-  // 64-wide tiles when they fit in one wave, else 128-wide (a second partial
-  // wave costs more than the wider tile)
-  const int tiles64 = ceil_div(g.N, 64) * ceil_div(g.M, kBM);
-  if (tiles64 <= num_sms) return launch_bn<64, 4>(g, d_err, num_sms, s);
-  return launch_bn<128, 3>(g, d_err, num_sms, s);
+  // the narrowest tile that covers the product in one wave, else 256-wide
+  // tiles: a tcgen05.mma re-reads its whole 128-row A operand from shared
+  // memory for every BN columns, so wider tiles move fewer operand bytes per
+  // flop, while narrower ones spread a small product over more SMs
+  const int m_tiles = ceil_div(g.M, kBM);
+  if (ceil_div(g.N, 64) * m_tiles <= num_sms) return launch_bn<64, 4, 2>(g, d_err, num_sms, s);
+  if (ceil_div(g.N, 128) * m_tiles <= num_sms) return launch_bn<128, 3, 2>(g, d_err, num_sms, s);
+  return launch_bn<256, 4, 1>(g, d_err, num_sms, s);
 }
 
 }  // namespace kf

@@ -10,6 +10,12 @@ namespace kf {
 
 constexpr unsigned long long kWaitNs = 2000000000ull;   // bounded mbarrier waits
 
+// a 2-D TMA map over `rows` contiguous rows of `cols` bf16 (cols * 2 a
+// multiple of 16 and at most 128 bytes), boxes of box_rows whole rows,
+// 128-byte swizzle; false if the driver entry point is missing or the
+// arguments are refused
+bool encode_rows_map_bf16(CUtensorMap* m, const void* base, uint64_t rows, int cols, int box_rows);
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -18,6 +18,7 @@ SHAPES = [
     (1000, 200, 128),    # N not a multiple of the tile
     (200, 640, 320),     # odd number of 64-wide K blocks: a short last pipeline stage
     (4096, 768, 3072),   # large M
+    (2100, 2340, 768),   # 256-wide tiles with ragged M and N
 ]
 
 
