@@ -5,6 +5,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <string>
@@ -89,6 +90,7 @@ struct kf_ctx {
   int4* groups = nullptr;
   float* part_o = nullptr;
   float2* part_ml = nullptr;
+  int* split_count = nullptr;   // [max groups][H] split counters of the warp-MMA attention
   size_t part_units = 0;
   int* d_err = nullptr;
   // graphs
@@ -216,6 +218,19 @@ static void attn_plan(kf_ctx* c, int n_groups, int R, int max_keys, int* n_split
   *kps = round_up(ceil_div(c->cfg.max_len, s), 64);
 }
 
+// warp-MMA attention: split the keys only while the (group, head) CTAs
+// leave SMs idle, into at most 4 splits, and only into splits of more than
+// one tile (those CTAs merge their own splits; measured on OWT-shaped
+// decode: 1 and 8 sequences gain 10-14%, 32 and more lose with any split)
+static void attn_plan_mma(kf_ctx* c, int n_groups, int R, int* n_split, int* kps) {
+  const int L = c->cfg.max_len;
+  const int ctas = n_groups * c->H;
+  int s = ctas >= c->num_sms ? 1 : std::min(4, ceil_div(c->num_sms, std::max(1, ctas)));
+  while (s > 1 && (round_up(ceil_div(L, s), kPage) <= 128 || (size_t)s * R * c->H > c->part_units)) --s;
+  *n_split = s;
+  *kps = round_up(ceil_div(L, s), kPage);
+}
+
 // L decoder layers over R rows (Table 4): pre-norm attention and MLP blocks.
 // On the fused tensor-core path (c->fused) the pre-norms run inside the
 // GEMMs: xn holds bf16(x), ss the per-64-column sums of squares written by
@@ -233,7 +248,8 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   const bool tc_attn = c->fused && rows > 8 && (c->cfg.flags & KF_FLAG_TC_ATTN);
   const bool mma_attn = !tc_attn && attention_mma_supported(c->bf16, c->hd, rows);
   int n_split, kps;
-  attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
+  if (mma_attn) attn_plan_mma(c, n_groups, R, &n_split, &kps);
+  else attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
   auto norm_in = [&](Epi& e) {
     e.ss_in = c->ss; e.nslot = d / 64; e.inv_d = 1.0f / d; e.eps = c->cfg.rms_eps;
   };
@@ -273,14 +289,16 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     a.len = groups ? nullptr : c->d_len;   // decode: keys below it are stable during the step
+    a.split_count = c->split_count;
     prof_begin(c, KF_KIND_ATTENTION);
+    bool merged = false;
     if (tc_attn) launch_attention_tc(a, n_groups, s);
     else if (mma_attn) {
-      if (launch_attention_mma(a, n_groups, rows, c->cfg.max_len, s) != 0) c->launch_failed = true;
+      if (launch_attention_mma(a, n_groups, rows, c->cfg.max_len, s, &merged) != 0) c->launch_failed = true;
     }
     else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
     prof_end(c);
-    if (n_split > 1) {
+    if (n_split > 1 && !merged) {
       prof_begin(c, KF_KIND_ATTN_COMBINE);
       launch_attn_combine(c->bf16, a, s);
       prof_end(c);
@@ -611,7 +629,8 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
     c->part_units = std::max(c->part_units, (size_t)ceil_div(cfg.max_len, attention_tc_max_keys()) *
                                                 c->R_cap * c->H);
   if ((r = dalloc(c, &c->part_o, c->part_units * c->hd * 4)) ||
-      (r = dalloc(c, &c->part_ml, c->part_units * sizeof(float2))))
+      (r = dalloc(c, &c->part_ml, c->part_units * sizeof(float2))) ||
+      (r = dalloc(c, &c->split_count, (size_t)std::max(R, cfg.max_batch) * c->H * sizeof(int))))
     return bail(r);
   e = cudaDeviceSynchronize();
   if (e != cudaSuccess) { cuda_fail(c, e, "init"); return bail(KF_E_CUDA); }

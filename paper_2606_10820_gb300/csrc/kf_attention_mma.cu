@@ -44,13 +44,64 @@ constexpr int kQRows = 16;     // MMA M: query rows of the group, zero-padded
 constexpr int kPageBytes = kPage * kHD * 2;                  // one page of K (or V) of one head
 constexpr int kTileBytes = kTile * kHD * 2;                  // 16 KB
 
-// [NBUF K tiles][NBUF V tiles][Q 16 x 64][NBUF mbarriers][page ids], from a
+// [NBUF K tiles][NBUF V tiles][Q 16 x 64][NBUF mbarriers][flag][page ids], from a
 // 1024-byte aligned base (the swizzle pattern repeats every 8 rows)
 constexpr size_t smem_bytes(int nbuf, int pg_cap) {
-  return 1024 + (size_t)2 * nbuf * kTileBytes + (size_t)kQRows * kHD * 2 + 8 * nbuf + 4 * pg_cap;
+  return 1024 + (size_t)2 * nbuf * kTileBytes + (size_t)kQRows * kHD * 2 + 8 * nbuf + 8 + 4 * pg_cap;
 }
 
 }  // namespace
+
+// the split merge of one (group, head), by thread t: row t / 8, dims
+// 8 (t % 8) .. +7
+__device__ __forceinline__ void merge_splits(const float* part_o, const float2* part_ml, __nv_bfloat16* out,
+                                          int n_split, int R, int H, int row0, int nr, int h, int t) {
+  const int r = t >> 3, d0 = (t & 7) * 8;
+  if (r < nr) {
+    // one pass in split order, four splits' loads in flight at a time;
+    // the running maximum M rescales the sums when it grows
+    const int row = row0 + r;
+    float M = -INFINITY, L = 0.f, acc[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+    for (int sp0 = 0; sp0 < n_split; sp0 += 4) {
+      float2 ml[4];
+      float4 u0[4], u1[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (sp0 + j < n_split) {
+          const size_t u = ((size_t)(sp0 + j) * R + row) * H + h;
+          ml[j] = __ldcg(part_ml + u);
+          const float4* po = reinterpret_cast<const float4*>(part_o + u * kHD + d0);
+          u0[j] = __ldcg(po);
+          u1[j] = __ldcg(po + 1);
+        } else {
+          ml[j] = make_float2(-INFINITY, 0.f);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (ml[j].x == -INFINITY) continue;        // an empty split
+        const float Mn = fmaxf(M, ml[j].x);
+        const float cs = (M == -INFINITY) ? 0.f : expf(M - Mn);
+        const float w = expf(ml[j].x - Mn);
+        M = Mn;
+        L = L * cs + ml[j].y * w;
+        acc[0] = acc[0] * cs + u0[j].x * w; acc[1] = acc[1] * cs + u0[j].y * w;
+        acc[2] = acc[2] * cs + u0[j].z * w; acc[3] = acc[3] * cs + u0[j].w * w;
+        acc[4] = acc[4] * cs + u1[j].x * w; acc[5] = acc[5] * cs + u1[j].y * w;
+        acc[6] = acc[6] * cs + u1[j].z * w; acc[7] = acc[7] * cs + u1[j].w * w;
+      }
+    }
+    const float inv = 1.f / L;
+    uint4 pk;
+    pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+    pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+    pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+    pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+    *reinterpret_cast<uint4*>(out + (size_t)row * H * kHD + h * kHD + d0) = pk;
+  }
+}
 
 // NBUF = 1: CTAs of at most one key tile; NBUF = 2: two tile buffers.  TWO:
 // groups of more than 8 rows (rows 8..15 of the MMA carry data).  Decode
@@ -69,7 +120,7 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
   __nv_bfloat16* Vs = Ks + NBUF * kTile * kHD;                // [NBUF][128][64] swizzled
   __nv_bfloat16* Qs = Vs + NBUF * kTile * kHD;                // [16][64] swizzled
   uint64_t* bars = reinterpret_cast<uint64_t*>(Qs + kQRows * kHD);
-  int* s_pg = reinterpret_cast<int*>(bars + NBUF);            // [a.pg_cap] (NBUF = 2)
+  int* s_pg = reinterpret_cast<int*>(bars + NBUF) + 2;       // [a.pg_cap] (NBUF = 2), after a flag
 
   const int gi = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
   const bool early = a.len != nullptr && a.groups == nullptr;
@@ -373,6 +424,24 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
       }
     }
   }
+  if constexpr (NBUF > 1) {
+    // the last split CTA of this (group, head) to finish merges the
+    // partials in split order (the same result whichever CTA it is) and
+    // re-arms the counter for the next launch
+    if (a.split_count == nullptr) return;
+    int* s_last = s_pg - 2;
+    __threadfence();
+    __syncthreads();
+    int* cnt = a.split_count + (size_t)gi * a.H + h;
+    if (t == 0) *s_last = atomicAdd(cnt, 1) == a.n_split - 1;
+    __syncthreads();
+    if (*s_last) {
+      __threadfence();
+      merge_splits(a.part_o, a.part_ml, reinterpret_cast<__nv_bfloat16*>(a.out), a.n_split, a.R, a.H, row0,
+                   nr, h, t);
+      if (t == 0) *cnt = 0;
+    }
+  }
 }
 
 template <int NBUF, bool TWO>
@@ -388,10 +457,16 @@ static void launch_nb(const CUtensorMap& map, const AttnArgs& a, int n_groups, c
 
 bool attention_mma_supported(bool bf16, int hd, int rows) { return bf16 && hd == kHD && rows <= kQRows; }
 
-int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_keys, cudaStream_t s) {
+int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_keys, cudaStream_t s,
+                         bool* merged) {
+  *merged = false;
   if (n_groups == 0) return 0;
   AttnArgs a = a0;
   const int keys = std::min(a.keys_per_split, max_keys);   // the most keys of one CTA
+  // CTAs of several tiles merge their own splits; single-tile CTAs (6 per
+  // SM, 80 registers) leave it to k_attn_combine
+  if (keys <= kTile || a.n_split == 1) a.split_count = nullptr;
+  *merged = a.split_count != nullptr;
   a.pg_cap = ceil_div(keys, kPage);
   // this layer's K/V pages as rows of 64 bf16: ((page * 2 + kv) * H + head) * 16 + key
   const size_t layer_elems = (size_t)a.n_pages * 2 * a.H * kPage * kHD;

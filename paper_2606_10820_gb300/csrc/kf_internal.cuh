@@ -380,6 +380,8 @@ struct AttnArgs {
   const int32_t* len = nullptr;  // decode: committed length per sequence (keys below it are
                                  // not written during the step), or NULL
   int pg_cap = 0;                // pages of one CTA's key range (set by the launcher)
+  int* split_count = nullptr;    // [groups][H] zeroed counters: the warp-MMA kernel merges
+                                 // its own splits (no k_attn_combine launch)
 };
 // max_keys: the most keys any row of the launch can see (max_len bound)
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
@@ -387,7 +389,9 @@ void launch_attn_combine(bool bf16, const AttnArgs& a, cudaStream_t s);
 // decode attention on warp-level MMA (bf16 cache, head_dim 64, <= 16 rows per
 // group; rows: the most rows of any group); -1 if the TMA map is refused
 bool attention_mma_supported(bool bf16, int hd, int rows);
-int launch_attention_mma(const AttnArgs& a, int n_groups, int rows, int max_keys, cudaStream_t s);
+// *merged: the kernel merged its key splits itself (no k_attn_combine needed)
+int launch_attention_mma(const AttnArgs& a, int n_groups, int rows, int max_keys, cudaStream_t s,
+                         bool* merged);
 // tensor-core decode attention (bf16 cache, head_dim 64, <= 16 rows per group,
 // keys_per_split <= attention_tc_max_keys())
 void launch_attention_tc(const AttnArgs& a, int n_groups, cudaStream_t s);

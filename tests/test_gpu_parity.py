@@ -341,6 +341,20 @@ def test_owt_ragged_paged(kf):
     dec.close()
 
 
+def test_owt_small_batch_split_keys(kf):
+    """Two sequences of a 1024-position model: the attention splits each
+    sequence's keys over 4 CTAs (256 keys each) and merges the partial
+    softmaxes in the kernel; the 300-token prompt leaves its last split
+    empty."""
+    cfg = OWT.replace(n_layer=2)
+    w = make_weights(cfg)
+    prompts = make_prompts([300, 700], cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 0, 4], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
+
+
 def _sampled(kf, cfg, w, prompts, pick, ks, max_k, seed):
     """Full batch on the GPU (graph replay), the oracle on sampled sequences."""
     B = len(prompts)
