@@ -9,7 +9,9 @@
 // copy per page and operand lands it 128-byte swizzled (16-byte chunk c of
 // row r at chunk c ^ (r % 8)), so ldmatrix reads are conflict-free, and one
 // mbarrier per buffer counts the bytes.  NBUF = 2: a ring of two buffers,
-// the next tile in flight while one is reduced.  Warp w owns keys
+// the next tile in flight while one is reduced (3 CTAs per SM); NBUF = 1:
+// one buffer refilled after each tile, 6 CTAs per SM overlapping each
+// other's loads.  Warp w owns keys
 // 32w .. 32w+31 of every tile and keeps its own online softmax over them
 // (FlashAttention-2 style):
 //   S = Q K^T      16 rows x 32 keys, 16 MMAs (Q zero-padded to 16 rows)
@@ -103,7 +105,7 @@ __device__ __forceinline__ void merge_splits(const float* part_o, const float2* 
   }
 }
 
-// NBUF = 1: CTAs of at most one key tile; NBUF = 2: two tile buffers.  TWO:
+// NBUF = 1: one tile buffer, refilled after each tile; NBUF = 2: two tile buffers.  TWO:
 // groups of more than 8 rows (rows 8..15 of the MMA carry data).  Decode
 // CTAs (a.len set, one group per sequence): the pages wholly before the
 // sequence's committed length were written by earlier steps and the page
@@ -145,12 +147,7 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int g = lane >> 2, tq = lane & 3;     // MMA fragment row group / column pair
 
-  int n_tiles = k_end > k_begin ? ceil_div(k_end - k_begin, kTile) : 0;
-  if (NBUF == 1 && n_tiles > 1) {
-    // the single-buffer variant is launched only for CTAs of at most one tile
-    if (t == 0) atomicOr(a.d_err, kErrInternal);
-    n_tiles = 1;
-  }
+  const int n_tiles = k_end > k_begin ? ceil_div(k_end - k_begin, kTile) : 0;
   const int pg0 = k_begin / kPage;            // k_begin is a multiple of the page size
   int n_pg = 0;
   if constexpr (NBUF > 1) {
@@ -463,19 +460,33 @@ int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_key
   if (n_groups == 0) return 0;
   AttnArgs a = a0;
   const int keys = std::min(a.keys_per_split, max_keys);   // the most keys of one CTA
-  // CTAs of several tiles merge their own splits; single-tile CTAs (6 per
-  // SM, 80 registers) leave it to k_attn_combine
-  if (keys <= kTile || a.n_split == 1) a.split_count = nullptr;
+  static int num_sms = 0;
+  if (!num_sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
+  }
+  const bool two = rows > 8;
+  const long ctas = (long)n_groups * a.H * a.n_split;
+  // two buffers (3 CTAs per SM) only while the CTAs fit in one wave of
+  // them; otherwise one buffer (6 per SM, 5 with 16-row groups; a CTA of
+  // several tiles refills it after each), twice the CTAs in flight.
+  // Measured on OWT-shaped decode at k = 4: batch 128 401k -> 423k, batch
+  // 256 481k -> 493k tokens/s; batch 32 (384 CTAs) 239k with two buffers,
+  // 209k with one
+  const bool one = keys <= kTile || ctas > 3L * num_sms;
+  // CTAs with two buffers merge their own splits; single-buffer CTAs (80
+  // registers) leave it to k_attn_combine
+  if (one || a.n_split == 1) a.split_count = nullptr;
   *merged = a.split_count != nullptr;
-  a.pg_cap = ceil_div(keys, kPage);
+  a.pg_cap = one ? 0 : ceil_div(keys, kPage);   // staged page ids (two-buffer CTAs)
   // this layer's K/V pages as rows of 64 bf16: ((page * 2 + kv) * H + head) * 16 + key
   const size_t layer_elems = (size_t)a.n_pages * 2 * a.H * kPage * kHD;
   CUtensorMap map;
   if (!encode_rows_map_bf16(&map, static_cast<const __nv_bfloat16*>(a.kv) + (size_t)a.layer * layer_elems,
                             (uint64_t)a.n_pages * 2 * a.H * kPage, kHD, kPage))
     return -1;
-  const bool two = rows > 8;
-  if (keys <= kTile) {
+  if (one) {
     if (two) launch_nb<1, true>(map, a, n_groups, s);
     else launch_nb<1, false>(map, a, n_groups, s);
   } else {
