@@ -13,6 +13,7 @@ SHAPES = [
     (130, 384, 768),     # ragged M across two row tiles
     (64, 768, 3072),     # AR-step MLP-down shape, deep split-K
     (512, 2304, 768),    # LM1B k=4 QKV
+    (512, 768, 3072),    # LM1B k=4 MLP-down: 128-wide tiles, split-K 4
     (320, 3072, 768),    # first-step rows (P=1), MLP-up
     (256, 30720, 768),   # LM-head shape (vocab padded to 256)
     (1000, 200, 128),    # N not a multiple of the tile
