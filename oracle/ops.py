@@ -30,7 +30,8 @@ def gelu_tanh(x: np.ndarray) -> np.ndarray:
     reading: the tanh form 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3)))
     for both the backbone MLP and the noise encoder.
     """
-    c = np.sqrt(2.0 / np.pi)
+    x = np.asarray(x)
+    c = x.dtype.type(np.sqrt(2.0 / np.pi))      # a constant of x's own type
     return 0.5 * x * (1.0 + np.tanh(c * (x + 0.044715 * x * x * x)))
 
 
@@ -69,7 +70,7 @@ def causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray,
     Scale 1/sqrt(hd).
     """
     hd = q.shape[-1]
-    scores = np.einsum("nhd,mhd->hnm", q, k) / np.sqrt(hd)
+    scores = np.einsum("nhd,mhd->hnm", q, k) / q.dtype.type(np.sqrt(hd))
     mask = np.asarray(k_pos)[None, :] > np.asarray(q_pos)[:, None]    # [n, m]
     scores = np.where(mask[None, :, :], -np.inf, scores)
     scores = scores - scores.max(axis=-1, keepdims=True)
