@@ -52,9 +52,6 @@ extern "C" {
 #define KF_FLAG_NO_GRAPH 1       /* launch kernels eagerly instead of replaying a CUDA graph */
 #define KF_FLAG_SIMT_GEMM 2      /* bf16 mode: use the SIMT GEMM, not tcgen05   */
 #define KF_FLAG_NO_PDL 4         /* launch without programmatic dependent launch */
-#define KF_FLAG_TC_ATTN 8        /* bf16, head_dim 64: attention of groups of more than 8
-                                    query rows on the tcgen05 kernel instead of the
-                                    warp-MMA kernel (kept for comparison)        */
 
 /*
  * Model and runtime configuration.  Table 4 gives the backbone (pre-norm
@@ -132,8 +129,14 @@ int kf_init(const kf_config* cfg, const kf_weights* w, void* stream,
  * concatenation of the B prompts (host or device, int32 ids in [0, V)),
  * lens[b] >= 1 their lengths (host).  The KV of every prompt token but the
  * last is computed and cached; the last token of each prompt becomes its one
- * pending token.  Any earlier batch is dropped.  Errors: KF_E_ARG,
- * KF_E_CAPACITY (a prompt is longer than max_len - 1, or the pool is full).
+ * pending token.  Any earlier batch is dropped, and the context's device
+ * error word is cleared (collect earlier asynchronous errors with kf_sync
+ * first).  Synchronises.  Host prompts are range-checked before any launch
+ * (KF_E_ARG); device-resident prompts are checked by the embedding kernel:
+ * an id outside [0, V) is embedded as id 0, flags the error word, and the
+ * call returns KF_E_DEVICE (the batch is then unusable until the next
+ * kf_prefill).  Errors: KF_E_ARG, KF_E_CAPACITY (a prompt is longer than
+ * max_len - 1, or the pool is full), KF_E_CUDA, KF_E_DEVICE.
  */
 int kf_prefill(kf_ctx* ctx, int32_t B, const int32_t* tokens,
                const int32_t* lens);
@@ -153,7 +156,12 @@ int kf_prefill(kf_ctx* ctx, int32_t B, const int32_t* tokens,
  * Afterwards each sequence's cache holds P more tokens and the emitted tokens
  * are its pending tokens (fixed stride, App. C.1).  B must equal the prefilled
  * batch and k <= max_k.  Errors: KF_E_ARG, KF_E_STATE, KF_E_CAPACITY,
- * KF_E_CUDA, KF_E_DEVICE (only reported by calls that synchronise).
+ * KF_E_CUDA, KF_E_DEVICE.  A call with host out_tokens synchronises and
+ * reports the device error word; with device out_tokens it returns after
+ * enqueueing, and kf_sync reports the word.  Once a kernel has flagged an
+ * error (a bounded wait ran out, an invalid page or token id), the token
+ * map writes -1 for every slot of that and every later step until the next
+ * kf_prefill.
  */
 int kf_decode_step(kf_ctx* ctx, int32_t B, int32_t k, const float* noise,
                    int32_t* out_tokens);

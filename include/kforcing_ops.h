@@ -21,8 +21,11 @@ extern "C" {
  * backbone (Table 4: QKV, O, MLP) and the LM head are this contraction.
  * A, W: bf16, row-major, rows 16-byte aligned; K a multiple of 64 for
  * KF_GEMM_TCGEN05, N a multiple of 4.  out: fp32 row-major [M][N].  The first
- * call allocates a 4-byte device error word that lives until process exit.
- * Errors: KF_E_ARG (shapes / alignment), KF_E_CUDA.
+ * call on a device allocates a 4-byte device error word for that device that
+ * lives until process exit; each call clears it on `stream` before its
+ * kernel runs, and the kernel ORs its error bits into it (a bounded
+ * pipeline wait that ran out).  Asynchronous: kf_op_status(stream) reports
+ * those errors.  Errors: KF_E_ARG (shapes / alignment), KF_E_CUDA.
  */
 int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, const void* A, const void* W,
                     float* out, void* stream);
@@ -40,8 +43,14 @@ int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, const void* A
  * aligned rows, d a multiple of 64; noise: fp32 [rows] in [0,1);
  * tokens: int32 [rows].  All device pointers.  The record scratch
  * (rows x ceil(V/32) x 16 bytes) is allocated with cudaMalloc on first use
- * and grown when a call needs more; it lives until process exit, and calls
- * that overlap on the GPU share it.  Errors: KF_E_ARG, KF_E_OOM, KF_E_CUDA.
+ * on each device and grown when a call needs more (growth first waits for
+ * the whole device); it lives until process exit.  Host threads are
+ * serialised around the buffer, but calls whose work overlaps on the GPU
+ * (several streams) share it and race.  Asynchronous: the call clears the
+ * device's op error word on `stream`; when a kernel of the call flags an
+ * error (a bounded wait ran out, so records may be stale) every token is -1
+ * and kf_op_status(stream) returns KF_E_DEVICE.
+ * Errors: KF_E_ARG, KF_E_OOM, KF_E_CUDA.
  */
 int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const void* w_head,
                       const float* noise, float tau, int32_t map_kind, int32_t* tokens,
@@ -64,12 +73,25 @@ int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const v
  * array's device address (cudaGetSymbolAddress); make that first call before
  * any stream capture.  All calls share the one array: calls whose work
  * overlaps on the GPU (different streams, or other threads) race on it.
+ * Its error word is also static and cleared at the start of each call; when
+ * a kernel of the call flags an error every token is -1, and
+ * kf_op_status(stream) reports it without allocating.
  * Arguments, layouts and the other errors are those of kf_op_head_tokens.
  */
 #define KF_NOALLOC_MAX_RECORDS 262144
 int kf_op_head_tokens_noalloc(int32_t rows, int32_t V, int32_t d, const void* x,
                               const void* w_head, const float* noise, float tau,
                               int32_t map_kind, int32_t* tokens, void* stream);
+
+/*
+ * Device errors of the entry points above on the current device: waits for
+ * `stream`, then reads and clears the error word of the allocating entries
+ * (the last kf_op_gemm_bf16 / kf_op_head_tokens call on this device) and the
+ * static one of kf_op_head_tokens_noalloc (its last call).  Returns KF_OK,
+ * KF_E_DEVICE when a kernel flagged an error (kf_last_error(NULL) gives the
+ * bits), or KF_E_CUDA.  Allocates nothing.
+ */
+int kf_op_status(void* stream);
 
 /*
  * Training-time attention of K-Forcing (App. C.2): SingleForward (blocks = 1)

@@ -241,15 +241,12 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   const int d = c->d, H = c->H, F = c->F;
   cudaStream_t s = c->stream;
   // Attention: the warp-MMA kernel for the bf16 cache with head_dim 64; the
-  // tcgen05 kernel for groups of more than 8 rows only on request
-  // (KF_FLAG_TC_ATTN, measured slower); the FP32-FMA kernel otherwise (fp32
-  // cache, head_dim 32).
+  // FP32-FMA kernel otherwise (fp32 cache, head_dim 32).
   const int rows = groups ? kMaxGroupRows : uniform_rows;
-  const bool tc_attn = c->fused && rows > 8 && (c->cfg.flags & KF_FLAG_TC_ATTN);
-  const bool mma_attn = !tc_attn && attention_mma_supported(c->bf16, c->hd, rows);
+  const bool mma_attn = attention_mma_supported(c->bf16, c->hd, rows);
   int n_split, kps;
   if (mma_attn) attn_plan_mma(c, n_groups, R, &n_split, &kps);
-  else attn_plan(c, n_groups, R, tc_attn ? attention_tc_max_keys() : (1 << 30), &n_split, &kps);
+  else attn_plan(c, n_groups, R, 1 << 30, &n_split, &kps);
   auto norm_in = [&](Epi& e) {
     e.ss_in = c->ss; e.nslot = d / 64; e.inv_d = 1.0f / d; e.eps = c->cfg.rms_eps;
   };
@@ -292,8 +289,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.split_count = c->split_count;
     prof_begin(c, KF_KIND_ATTENTION);
     bool merged = false;
-    if (tc_attn) launch_attention_tc(a, n_groups, s);
-    else if (mma_attn) {
+    if (mma_attn) {
       if (launch_attention_mma(a, n_groups, rows, c->cfg.max_len, s, &merged) != 0) c->launch_failed = true;
     }
     else launch_attention(c->bf16, a, n_groups, c->cfg.max_len, s);
@@ -380,7 +376,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   prof_begin(c, KF_KIND_HEAD_SELECT);
   launch_head_select(c->bf16, B * nout, c->rec, c->nchunk, c->head_in, d, mtp ? c->w_mtp : c->w_head,
                      c->V, 1.0f / c->cfg.tau, c->cfg.map_kind, noise, c->tokens, mtp ? B : 0,
-                     (size_t)c->V_pad * d, s);
+                     (size_t)c->V_pad * d, c->d_err, s);
   prof_end(c);
   prof_begin(c, KF_KIND_COMMIT);
   launch_commit(B, P, k, c->tokens, c->d_pending, c->pend_stride, c->d_len, s);
@@ -622,12 +618,8 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
       (r = dalloc(c, &c->head_map, (size_t)c->NR_cap * 4)) ||
       (r = dalloc(c, &c->groups, (size_t)R * sizeof(int4))) || (r = dalloc(c, &c->d_err, 4)))
     return bail(r);
-  // split-KV partials: small batches split to fill the SMs; the tensor-core
-  // attention also splits every context longer than its per-CTA key limit
+  // split-KV partials: small batches split to fill the SMs
   c->part_units = (size_t)4 * c->num_sms * kMaxGroupRows;
-  if (c->fused)
-    c->part_units = std::max(c->part_units, (size_t)ceil_div(cfg.max_len, attention_tc_max_keys()) *
-                                                c->R_cap * c->H);
   if ((r = dalloc(c, &c->part_o, c->part_units * c->hd * 4)) ||
       (r = dalloc(c, &c->part_ml, c->part_units * sizeof(float2))) ||
       (r = dalloc(c, &c->split_count, (size_t)std::max(R, cfg.max_batch) * c->H * sizeof(int))))
@@ -699,17 +691,23 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
     if (ln[b] + 1 > c->cfg.max_len) return fail(c, KF_E_CAPACITY, "prompt longer than max_len - 1");
     total += ln[b];
   }
+  // Host prompts are checked here; device-resident prompts are checked where
+  // the embedding kernel reads them (an id outside [0, V) embeds as id 0 and
+  // flags the device error word: the call then returns KF_E_DEVICE).
   std::vector<int32_t> tok(total);
-  if (is_device_ptr(tokens)) {
+  const bool dev_tok = is_device_ptr(tokens);
+  if (dev_tok) {
     KF_CUDA(cudaMemcpy(tok.data(), tokens, total * 4, cudaMemcpyDeviceToHost));
   } else {
     memcpy(tok.data(), tokens, total * 4);
+    for (size_t i = 0; i < total; ++i)
+      if (tok[i] < 0 || tok[i] >= c->V) return fail(c, KF_E_ARG, "token id out of range");
   }
-  for (size_t i = 0; i < total; ++i)
-    if (tok[i] < 0 || tok[i] >= c->V) return fail(c, KF_E_ARG, "token id out of range");
   KF_CUDA(cudaStreamSynchronize(c->stream));
   c->have_batch = false;
   c->have_step = false;
+  // a new batch starts with a clear device error word
+  KF_CUDA(cudaMemsetAsync(c->d_err, 0, 4, c->stream));
   reset_pages(c);
   for (int b = 0; b < B; ++b) {
     bool dirty = false;

@@ -358,12 +358,8 @@ __global__ void k_attn_combine(AttnArgs a) {
 template <typename TA, int HD, int R, int NBUF>
 static void launch_rb(const AttnArgs& a, int n_groups, cudaStream_t s) {
   const size_t smem = AttnSmem<TA, HD>::bytes(R, NBUF);
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(k_attention<TA, HD, R, NBUF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
-    attr = true;
-  }
+  static PerDevice attr;
+  set_smem_attr(attr, k_attention<TA, HD, R, NBUF>, smem);
   dim3 grid(n_groups, a.H, a.n_split);
   kf_launch(k_attention<TA, HD, R, NBUF>, grid, dim3(kAttnThreads), smem, s, a);
 }

@@ -443,12 +443,9 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
 
 template <int NBUF, bool TWO>
 static void launch_nb(const CUtensorMap& map, const AttnArgs& a, int n_groups, cudaStream_t s) {
-  static size_t attr = 0;
+  static PerDevice attr;
   const size_t smem = smem_bytes(NBUF, a.pg_cap);
-  if (smem > attr) {
-    cudaFuncSetAttribute(k_attention_mma<NBUF, TWO>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    attr = smem;
-  }
+  set_smem_attr(attr, k_attention_mma<NBUF, TWO>, smem);
   kf_launch(k_attention_mma<NBUF, TWO>, dim3(n_groups, a.H, a.n_split), dim3(kThr), smem, s, map, a);
 }
 
@@ -460,12 +457,7 @@ int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_key
   if (n_groups == 0) return 0;
   AttnArgs a = a0;
   const int keys = std::min(a.keys_per_split, max_keys);   // the most keys of one CTA
-  static int num_sms = 0;
-  if (!num_sms) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
-  }
+  const int num_sms = device_sms();
   const bool two = rows > 8;
   const long ctas = (long)n_groups * a.H * a.n_split;
   // two buffers (3 CTAs per SM) only while the CTAs fit in one wave of

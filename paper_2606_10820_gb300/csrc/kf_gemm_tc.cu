@@ -479,16 +479,10 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
   const size_t smem = (size_t)STAGES * AT * (MT * kBM * kBK * 2 + BN * kBK * 2) + 1024 + 256 + sizeof(EpiMeta);
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, EPI, MT, AT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
-    attr_set = true;
-  }
-  // a cluster of `splits` CTAs must fit on one GPC
-  static int max_cluster = 0;
-  if (!max_cluster) {
-    max_cluster = 1;
+  static PerDevice attr, cluster;
+  set_smem_attr(attr, k_gemm_tc<BN, STAGES, EPI, MT, AT>, smem);
+  // the largest cluster of these CTAs that fits on one GPC of this device
+  const int max_cluster = (int)per_device(cluster, [&] {
     for (int cs = 8; cs > 1; --cs) {
       cudaLaunchConfig_t q = {};
       q.gridDim = dim3(1, 1, cs);
@@ -500,13 +494,12 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
       q.attrs = &ca;
       q.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<BN, STAGES, EPI, MT, AT>, &q) == cudaSuccess && n > 0) {
-        max_cluster = cs;
-        break;
-      }
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<BN, STAGES, EPI, MT, AT>, &q) == cudaSuccess && n > 0)
+        return (long long)cs;
       cudaGetLastError();
     }
-  }
+    return 1ll;
+  });
   if (splits > max_cluster) {
     splits = max_cluster;
     kbps = ceil_div(kb_total, splits);
@@ -557,12 +550,7 @@ static int launch_bn(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s)
 }
 
 int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
-  static int num_sms = 0;
-  if (!num_sms) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev);
-  }
+  const int num_sms = device_sms();
   // LM-head records: 256-wide tiles; above 128 rows both M tiles of a row
   // pair in one CTA (each weight tile is streamed from HBM once per 256 rows)
   if (g.epi.kind == EPI_HEAD) {

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -25,6 +26,57 @@ constexpr int kErrBadRow = 8;
 constexpr int kErrInternal = 16;   // a launch invariant of the host plan did not hold
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// One-time setup per device (function attributes, occupancy limits and SM
+// counts belong to each device's context): per_device(pd, f) returns f()'s
+// value for the current device, computed on the first call made with that
+// device current.  Thread-safe; devices past kMaxDevices recompute each call.
+constexpr int kMaxDevices = 64;
+struct PerDevice {
+  std::mutex mu;
+  bool done[kMaxDevices] = {};
+  long long val[kMaxDevices] = {};
+};
+template <typename F>
+inline long long per_device(PerDevice& pd, F init) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    return init();
+  }
+  std::lock_guard<std::mutex> lock(pd.mu);
+  if (!pd.done[dev]) {
+    pd.val[dev] = init();
+    pd.done[dev] = true;
+  }
+  return pd.val[dev];
+}
+// the SM count of the current device
+inline int device_sms() {
+  static PerDevice pd;
+  return (int)per_device(pd, [] {
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return (long long)(n > 0 ? n : 1);
+  });
+}
+// raise a kernel's dynamic shared-memory limit to `bytes` on the current
+// device (once per device and size; thread-safe)
+template <typename K>
+inline void set_smem_attr(PerDevice& pd, K* kern, size_t bytes) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    cudaGetLastError();
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    return;
+  }
+  std::lock_guard<std::mutex> lock(pd.mu);
+  if (pd.val[dev] < (long long)bytes) {
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    pd.val[dev] = (long long)bytes;
+  }
+}
 __host__ __device__ inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
 
 // storage <-> fp32
@@ -392,10 +444,6 @@ bool attention_mma_supported(bool bf16, int hd, int rows);
 // *merged: the kernel merged its key splits itself (no k_attn_combine needed)
 int launch_attention_mma(const AttnArgs& a, int n_groups, int rows, int max_keys, cudaStream_t s,
                          bool* merged);
-// tensor-core decode attention (bf16 cache, head_dim 64, <= 16 rows per group,
-// keys_per_split <= attention_tc_max_keys())
-void launch_attention_tc(const AttnArgs& a, int n_groups, cudaStream_t s);
-int attention_tc_max_keys();
 
 // message for kf_last_error(NULL) (calls without a context)
 void set_global_error(const std::string& msg);
@@ -422,11 +470,13 @@ void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
                         void* kv, int layer, int n_pages, const int32_t* page_table, int max_pages,
                         int* d_err, cudaStream_t s);
 // mtp_rows = B > 0: n_rows = B k blocks in head-major order, head j's weights
-// at w_head + j head_stride (elements); 0: one block per row of head_in
+// at w_head + j head_stride (elements); 0: one block per row of head_in.
+// err: the call's device error word (or NULL); when an earlier kernel set
+// it, every token is -1
 void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
                         int d, const void* w_head, int V, float inv_tau, int map_kind,
                         const float* noise, int32_t* tokens, int mtp_rows, size_t head_stride,
-                        cudaStream_t s);
+                        const int* err, cudaStream_t s);
 void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
                    int32_t* d_len, cudaStream_t s);
 

@@ -324,7 +324,7 @@ __global__ void __launch_bounds__(kSelThreads)
 k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
               const TA* __restrict__ w_head_all, int V, float inv_tau, int map_kind,
               const float* __restrict__ noise, int32_t* __restrict__ tokens, int mtp_rows,
-              size_t head_stride) {
+              size_t head_stride, const int* __restrict__ err) {
   pdl_trigger();
   pdl_wait();
   // one block per mapped row; MTP (mtp_rows = B > 0): block j B + b is head j
@@ -338,6 +338,14 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
     hrow = b;
     zrow = b * kk + j;
     w_head = w_head_all + (size_t)j * head_stride;
+  }
+  // an earlier kernel of the call flagged an error (e.g. a bounded wait ran
+  // out, so the records may be stale): token -1 instead of a stale choice.
+  // Every earlier kernel has completed (pdl_wait), so all threads read the
+  // same value.
+  if (err && *err) {
+    if (threadIdx.x == 0) tokens[zrow] = -1;
+    return;
   }
   const HeadRec* rec = rec_all + (size_t)row * nchunk;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -530,15 +538,15 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
 void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
                         int d, const void* w_head, int V, float inv_tau, int map_kind,
                         const float* noise, int32_t* tokens, int mtp_rows, size_t head_stride,
-                        cudaStream_t s) {
+                        const int* err, cudaStream_t s) {
   if (n_rows == 0) return;
   if (bf16)
     kf_launch(k_head_select<__nv_bfloat16>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk,
         (const __nv_bfloat16*)head_in, d, (const __nv_bfloat16*)w_head, V, inv_tau, map_kind,
-        noise, tokens, mtp_rows, head_stride);
+        noise, tokens, mtp_rows, head_stride, err);
   else
     kf_launch(k_head_select<float>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk, (const float*)head_in, d,
-        (const float*)w_head, V, inv_tau, map_kind, noise, tokens, mtp_rows, head_stride);
+        (const float*)w_head, V, inv_tau, map_kind, noise, tokens, mtp_rows, head_stride, err);
 }
 
 // ---------------------------------------------------------------- commit

@@ -8,14 +8,36 @@
 using namespace kf;
 
 namespace {
-int* g_err = nullptr;
-HeadRec* g_rec = nullptr;
-size_t g_rec_bytes = 0;
+// Scratch of the allocating entry points, per device: an error word (the
+// kernels OR their error bits into it; kf_op_status reads and clears it)
+// and the LM-head record buffer.  g_ops_mu guards both tables.
+struct OpScratch {
+  int* err = nullptr;
+  HeadRec* rec = nullptr;
+  size_t rec_bytes = 0;
+};
+OpScratch g_ops[kMaxDevices];
+std::mutex g_ops_mu;
 
-int ensure_err() {
-  if (g_err) return KF_OK;
-  if (cudaMalloc(&g_err, sizeof(int)) != cudaSuccess || cudaMemset(g_err, 0, sizeof(int)) != cudaSuccess)
+int current_device(int* dev) {
+  if (cudaGetDevice(dev) != cudaSuccess || *dev < 0 || *dev >= kMaxDevices) {
+    cudaGetLastError();
     return KF_E_CUDA;
+  }
+  return KF_OK;
+}
+
+// the current device's error word (allocated and zeroed on first use);
+// call with g_ops_mu held
+int ensure_err(int dev) {
+  if (g_ops[dev].err) return KF_OK;
+  int* e = nullptr;
+  if (cudaMalloc(&e, sizeof(int)) != cudaSuccess || cudaMemset(e, 0, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    if (e) cudaFree(e);
+    return KF_E_CUDA;
+  }
+  g_ops[dev].err = e;
   return KF_OK;
 }
 }  // namespace
@@ -33,7 +55,8 @@ static int head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const 
   g.epi.nchunk = nchunk;
   if (!tc_gemm_supported(g)) return KF_E_ARG;
   if (launch_gemm_tc(g, err, s) != 0) return KF_E_CUDA;
-  launch_head_select(true, rows, rec, nchunk, x, d, w_head, V, 1.0f / tau, map_kind, noise, tokens, 0, 0, s);
+  launch_head_select(true, rows, rec, nchunk, x, d, w_head, V, 1.0f / tau, map_kind, noise, tokens, 0, 0,
+                     err, s);
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
 }
 
@@ -53,8 +76,17 @@ extern "C" int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, co
   cudaStream_t s = (cudaStream_t)stream;
   if (impl == KF_GEMM_TCGEN05) {
     if (!tc_gemm_supported(g)) return KF_E_ARG;
-    if (ensure_err() != KF_OK) return KF_E_CUDA;
-    if (launch_gemm_tc(g, g_err, s) != 0) return KF_E_CUDA;
+    int dev = 0;
+    if (current_device(&dev) != KF_OK) return KF_E_CUDA;
+    int* err = nullptr;
+    {
+      std::lock_guard<std::mutex> lock(g_ops_mu);
+      if (ensure_err(dev) != KF_OK) return KF_E_CUDA;
+      err = g_ops[dev].err;
+    }
+    // each call starts with a clear error word (kf_op_status reads it)
+    if (cudaMemsetAsync(err, 0, sizeof(int), s) != cudaSuccess) return KF_E_CUDA;
+    if (launch_gemm_tc(g, err, s) != 0) return KF_E_CUDA;
   } else if (impl == KF_GEMM_SIMT) {
     launch_gemm_simt(true, g, s);
   } else {
@@ -67,24 +99,33 @@ extern "C" int kf_op_head_tokens(int32_t rows, int32_t V, int32_t d, const void*
                                  const void* w_head, const float* noise, float tau,
                                  int32_t map_kind, int32_t* tokens, void* stream) {
   if (!head_args_ok(rows, V, d, x, w_head, noise, tau, map_kind, tokens)) return KF_E_ARG;
-  if (ensure_err() != KF_OK) return KF_E_CUDA;
+  int dev = 0;
+  if (current_device(&dev) != KF_OK) return KF_E_CUDA;
+  cudaStream_t s = (cudaStream_t)stream;
   const size_t need = (size_t)rows * ceil_div(V, kChunk) * sizeof(HeadRec);
-  if (need > g_rec_bytes) {
-    cudaStream_t s = (cudaStream_t)stream;
-    if (g_rec) {
-      cudaStreamSynchronize(s);   // a pending call may still read the old buffer
-      cudaFree(g_rec);
-      g_rec = nullptr;
-      g_rec_bytes = 0;
+  // The lock covers the buffer's growth and the launches that use it, so two
+  // host threads never free a buffer the other is about to launch on.  Work
+  // already enqueued on another stream may still read an old buffer: growth
+  // waits for the whole device first.
+  std::lock_guard<std::mutex> lock(g_ops_mu);
+  if (ensure_err(dev) != KF_OK) return KF_E_CUDA;
+  OpScratch& sc = g_ops[dev];
+  if (need > sc.rec_bytes) {
+    if (sc.rec) {
+      if (cudaDeviceSynchronize() != cudaSuccess) return KF_E_CUDA;
+      cudaFree(sc.rec);
+      sc.rec = nullptr;
+      sc.rec_bytes = 0;
     }
-    if (cudaMalloc(&g_rec, need) != cudaSuccess) {
+    if (cudaMalloc(&sc.rec, need) != cudaSuccess) {
       cudaGetLastError();
+      sc.rec = nullptr;
       return KF_E_OOM;
     }
-    g_rec_bytes = need;
+    sc.rec_bytes = need;
   }
-  return head_tokens(rows, V, d, x, w_head, noise, tau, map_kind, tokens, g_rec, g_err,
-                     (cudaStream_t)stream);
+  if (cudaMemsetAsync(sc.err, 0, sizeof(int), s) != cudaSuccess) return KF_E_CUDA;
+  return head_tokens(rows, V, d, x, w_head, noise, tau, map_kind, tokens, sc.rec, sc.err, s);
 }
 
 // ------------------------------------------------- no-allocation variant
@@ -95,7 +136,6 @@ static __device__ __align__(256) HeadRec g_noalloc_rec[KF_NOALLOC_MAX_RECORDS];
 static __device__ __align__(256) int g_noalloc_err;
 
 namespace {
-constexpr int kMaxDevices = 64;
 struct NoAllocScratch {
   HeadRec* rec = nullptr;
   int* err = nullptr;
@@ -141,4 +181,44 @@ extern "C" int kf_op_head_tokens_noalloc(int32_t rows, int32_t V, int32_t d, con
   // need no clearing, every one this call reads it writes first)
   if (cudaMemsetAsync(sc.err, 0, sizeof(int), s) != cudaSuccess) return KF_E_CUDA;
   return head_tokens(rows, V, d, x, w_head, noise, tau, map_kind, tokens, sc.rec, sc.err, s);
+}
+
+// Reads and clears the error words of the op entry points on the current
+// device after `stream` finishes: the allocating entries' word (if one of
+// them has run on this device) and the no-allocation entry's static word.
+// Allocates nothing.
+extern "C" int kf_op_status(void* stream) {
+  int dev = 0;
+  if (current_device(&dev) != KF_OK) return KF_E_CUDA;
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) {
+    cudaGetLastError();
+    set_global_error("kf_op_status: the stream reported a CUDA error");
+    return KF_E_CUDA;
+  }
+  int bits = 0;
+  int* err = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_ops_mu);
+    err = g_ops[dev].err;
+  }
+  if (err) {
+    int v = 0;
+    if (cudaMemcpy(&v, err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemset(err, 0, sizeof(int)) != cudaSuccess)
+      return KF_E_CUDA;
+    bits |= v;
+  }
+  int v = 0;
+  const int zero = 0;
+  if (cudaMemcpyFromSymbol(&v, g_noalloc_err, sizeof(int)) != cudaSuccess ||
+      cudaMemcpyToSymbol(g_noalloc_err, &zero, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    return KF_E_CUDA;
+  }
+  bits |= v;
+  if (bits) {
+    set_global_error("kf_op_status: device error flags " + std::to_string(bits));
+    return KF_E_DEVICE;
+  }
+  return KF_OK;
 }

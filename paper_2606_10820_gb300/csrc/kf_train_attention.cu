@@ -304,11 +304,8 @@ extern "C" int kf_op_train_attention(int32_t blocks, int32_t B, int32_t H, int32
   TrainAttnArgs a{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kk),
                   static_cast<const __nv_bfloat16*>(v), out, N, k, blocks, (int)T, H, q_begin, q_end,
                   dense ? 1 : 0};
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(k_train_attention, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes());
-    attr = true;
-  }
+  static PerDevice attr;
+  set_smem_attr(attr, k_train_attention, smem_bytes());
   const dim3 grid(ceil_div(q_end - q_begin, kRows), H, B);
   kf_launch(k_train_attention, grid, dim3(kThr), smem_bytes(), (cudaStream_t)stream, a);
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
