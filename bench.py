@@ -8,8 +8,13 @@ HBM; ``e2e`` = the same through the C ABI with host noise and host tokens,
 host<->device copies inside the timed region.  The k = 1 AR teacher step
 (kf_decode_step with k = 0) is measured the same way for the speedup.
 
-Default workload: the LM1B-shaped model (12 L, d 768, 12 heads, MLP 3072,
-V 30522, bf16), batch 64, prompt 32 -> 128, k = 4 vs the AR step.
+Headline workload: the OWT-shaped model (12 L, d 768, 12 heads, MLP 3072,
+V 50257, bf16) serving batch 512 with ragged prompts of 128..896 tokens in
+16-token pages, 128 new tokens, k = 4 vs the AR step: the largest batch of
+the metric's range.  Every other configuration (LM1B-shaped batch 64,
+OWT-shaped batch 1..256, medium batch 256) is measured in the same run and
+reported under ``configs`` with its tokens/s per k, the k-vs-k=1 speedup and
+the step roofline fraction.
 ``--impl reference`` times the CPU oracle on a bounded sample instead.
 Launch with torchrun for N > 1: each rank runs an independent replica.
 """
@@ -39,21 +44,20 @@ def parse():
     p.add_argument("--steps", type=int, default=5)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="kforcing", choices=["kforcing", "reference"])
-    p.add_argument("--workload", default="lm1b")
+    p.add_argument("--workload", default="", help="headline workload (default: owt_paged)")
     p.add_argument("--batch", type=int, default=0)
     p.add_argument("--k", type=int, default=4)
     p.add_argument("--gen", type=int, default=0, help="tokens per sequence (0: workload)")
     p.add_argument("--no-cpu", action="store_true", help="skip the cpu_baseline leg")
     p.add_argument("--no-ar", action="store_true", help="skip the k=1 AR leg")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the other configurations (LM1B, OWT batch 1..256, medium)")
+    p.add_argument("--extra-only", default="",
+                   help="comma-separated workload names: measure only these other configurations")
     p.add_argument("--train-attention", action="store_true",
                    help="SingleForward / DoubleForward training attention (App. C.2)")
     p.add_argument("--serving", action="store_true",
                    help="the G* teacher call and continuous batching (LM1B, batch 64)")
-    p.add_argument("--sweep-only", default="",
-                   help="comma-separated workload names: run only these sweep configurations")
-    p.add_argument("--sweep", action="store_true",
-                   help="one line per configuration: OWT-shaped batch 1..256, OWT paged "
-                        "batch 512, medium batch 256 (k vs the AR step)")
     return p.parse_args()
 
 
@@ -92,30 +96,35 @@ def dist_init(n):
 # ------------------------------------------------------------------ roofline
 def kind_costs(model, B, P, k, ctx_lens):
     """Algorithmic bytes and flops per launch of each kernel kind for one
-    decode call of shape (B, P, k) whose sequences have ctx_lens cached."""
+    decode call of shape (B, P, k) whose sequences have ctx_lens cached.
+
+    Bytes count what the method must move through HBM: a projection's
+    weights (N K), the attention's K/V reads of the keys it visits, the LM
+    head's weights. Activations, logits and records are excluded: the method
+    does not need them in HBM.  Flops are 2 M N K per projection and 4 hd
+    per visible (query, key) pair and head."""
     d, F, V, H = model.d_model, model.d_ff, model.vocab, model.n_head
     hd = d // H
     e = 2 if model.dtype == "bf16" else 4
-    kz = 1 if (getattr(model, "mtp_k", 0) and k) else k     # noise rows per sequence
+    mtp = bool(getattr(model, "mtp_k", 0) and k)
+    kz = 1 if mtp else k            # noise rows per sequence
     R = B * (P + kz)
     nh = B * max(k, 1)
-    nchunk = -(-V // 32)
 
-    def gemm(M, N, K, out_bytes):
-        return {"bytes": N * K * e + M * K * e + out_bytes, "flops": 2.0 * M * N * K}
+    def gemm(M, N, K):
+        return {"bytes": N * K * e, "flops": 2.0 * M * N * K}
     keys = sum(int(c) + P + kz for c in ctx_lens)
     vis = sum(sum(int(c) + i + 1 for i in range(P + kz)) for c in ctx_lens)
-    head = gemm(nh, V, d, nh * nchunk * 16)
-    if kz != k:        # MTP: k heads over B rows
-        head = {"bytes": k * V * d * e + B * d * e + nh * nchunk * 16, "flops": 2.0 * nh * V * d}
+    head = gemm(nh, V, d)
+    if mtp:        # k untied heads over the B noise tokens
+        head = {"bytes": k * V * d * e, "flops": 2.0 * nh * V * d}
     return {
-        "gemm_qkv": gemm(R, 3 * d, d, R * 3 * d * e),
-        "gemm_o": gemm(R, d, d, 2 * R * d * 4),
-        "gemm_up": gemm(R, F, d, R * F * e),
-        "gemm_down": gemm(R, d, F, 2 * R * d * 4),
+        "gemm_qkv": gemm(R, 3 * d, d),
+        "gemm_o": gemm(R, d, d),
+        "gemm_up": gemm(R, F, d),
+        "gemm_down": gemm(R, d, F),
         "gemm_head": head,
-        "attention": {"bytes": keys * H * hd * 2 * e + R * d * 4 + R * d * e,
-                      "flops": 4.0 * vis * H * hd},
+        "attention": {"bytes": keys * H * hd * 2 * e, "flops": 4.0 * vis * H * hd},
     }
 
 
@@ -190,12 +199,13 @@ class Clocks:
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_rate(model, w, prompts, k, budget_s=12.0, max_calls=6):
+def cpu_oracle_rate(model, w, prompts, k, budget_s=12.0, max_calls=6, dtype=None):
     """Oracle tokens/s over a bounded sample: decode calls on the given
-    prompts until the time budget is spent."""
+    prompts until the time budget is spent (the prefill is not timed)."""
     import oracle
     from synth import make_noise
-    dec = oracle.OracleDecoder(oracle.OracleModel(model, w))
+    dt = dtype if dtype is not None else np.float64
+    dec = oracle.OracleDecoder(oracle.OracleModel(model, w, dtype=dt))
     dec.prefill(prompts)
     B = len(prompts)
     zs = make_noise(max_calls, B, k)
@@ -208,65 +218,125 @@ def cpu_oracle_rate(model, w, prompts, k, budget_s=12.0, max_calls=6):
     return toks / el, calls, el
 
 
-def cpu_threads():
+def host_cores():
+    return os.cpu_count() or 1
+
+
+ARM_PARTS = {"0xd4f": "Arm Neoverse V2", "0xd40": "Arm Neoverse V1", "0xd0c": "Arm Neoverse N1",
+             "0xd49": "Arm Neoverse N2"}
+
+
+def cpu_model():
+    import platform
     try:
-        from threadpoolctl import threadpool_info
-        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
-        if n:
-            return int(max(n))
-    except Exception:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                low = line.lower()
+                if low.startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+                if low.startswith("cpu part"):
+                    part = line.split(":", 1)[1].strip()
+                    return f"{ARM_PARTS.get(part, 'Arm part ' + part)} ({platform.machine()})"
+    except OSError:
         pass
-    return os.cpu_count()
+    return platform.processor() or platform.machine()
+
+
+def _cpu_child(argv):
+    """Child process of cpu_oracle_sample: its BLAS thread count was fixed by
+    the environment before numpy loaded.  Prints one JSON object."""
+    name, nseq, k, budget, max_calls = argv[0], int(argv[1]), int(argv[2]), float(argv[3]), int(argv[4])
+    from synth import WORKLOADS, make_weights, workload_prompts
+    wl = WORKLOADS[name]
+    model = wl.model
+    w = make_weights(model)
+    prompts = workload_prompts(wl)
+    # a seeded pick of nseq sequences of the batch, with their own prompts
+    pick = np.random.default_rng(6).choice(len(prompts), size=min(nseq, len(prompts)), replace=False)
+    sample = [prompts[i] for i in sorted(pick)]
+    r, calls, el = cpu_oracle_rate(model, w, sample, k, budget_s=budget, max_calls=max_calls,
+                                   dtype=np.float32)
+    print(json.dumps({"rate": r, "calls": calls, "elapsed": el, "seqs": len(sample),
+                      "ctx": [int(len(p)) for p in sample]}))
+    return 0
+
+
+def cpu_oracle_sample(name, k, threads, nseq=2, budget=10.0, max_calls=8):
+    """The fp32 oracle, as it stands, on `threads` host threads (numpy's BLAS
+    pool, fixed before numpy loads), in a separate process; decode calls of
+    k on `nseq` sequences of the workload after their prompts are cached."""
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(threads)
+    p = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-child", name, str(nseq),
+                        str(k), str(budget), str(max_calls)], capture_output=True, text=True, env=env,
+                       timeout=900)
+    if p.returncode != 0:
+        raise RuntimeError("cpu oracle child failed: " + p.stderr[-2000:])
+    return json.loads(p.stdout.strip().splitlines()[-1])
+
+
+def cpu_baseline(name, k, B):
+    """fp32 oracle at 1 thread and at all host threads (reported, not a target)."""
+    n = host_cores()
+    one = cpu_oracle_sample(name, k, 1)
+    alln = cpu_oracle_sample(name, k, n)
+    return {"value": alln["rate"], "unit": "tokens/s", "cores": n, "kind": "oracle",
+            "cpu": cpu_model(),
+            "single_thread": {"value": one["rate"], "unit": "tokens/s", "cores": 1},
+            "sample": f"{alln['seqs']} of the {B} sequences (prompts {alln['ctx']}), "
+                      f"{alln['calls']} decode calls of k={k} after the prompt, numpy fp32, "
+                      f"{alln['elapsed']:.1f} s on {n} threads; {one['calls']} calls, "
+                      f"{one['elapsed']:.1f} s on 1 thread"}
 
 
 # ------------------------------------------------------------------ main
 def bench_config(w, B, gen, k):
     """The `config` object of the bench line (both arms)."""
     model = w.model
+    prompt = f"{w.prompt_len}" if not w.ragged else f"ragged {list(w.ragged)}"
     return {"workload": f"{w.name}: {model.n_layer}L d{model.d_model} H{model.n_head} "
-                        f"F{model.d_ff} V{model.vocab}, batch {B}, prompt "
-                        f"{w.prompt_len or 'ragged'} +{gen} tokens, k={k}",
+                        f"F{model.d_ff} V{model.vocab}, batch {B}, prompt {prompt} +{gen} tokens, k={k}",
             "batch": B, "k": k, "gen_tokens_per_seq": gen,
             "calls_per_step": -(-gen // max(k, 1)), "map": model.map,
-            "l2": "working set larger than L2 (weights + KV), no flush"}
+            "l2": "inputs larger than L2 (weights + KV pages), no flush"}
+
+
+HEADLINE = ("owt_paged", 512, 4)
 
 
 def workload_of(args):
     from synth import WORKLOADS
-    w = WORKLOADS[args.workload]
-    B = args.batch or w.batch
+    name = args.workload or HEADLINE[0]
+    w = WORKLOADS[name]
+    B = args.batch or (HEADLINE[1] if name == HEADLINE[0] else w.batch)
     gen = args.gen or w.gen_len
     return w, B, gen
 
 
 def run_reference(args):
     """The reference arm: the CPU oracle, as it stands, on the same workload."""
-    from synth import make_weights, workload_prompts
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     w, B, gen = workload_of(args)
-    model = w.model
-    weights = make_weights(model)
-    Bs = min(B, 16)
-    prompts = workload_prompts(w, Bs)
-    rates = []
-    for _ in range(max(1, args.warmup and 1)):
-        cpu_oracle_rate(model, weights, prompts, args.k, budget_s=5.0, max_calls=2)
-    t_all = time.perf_counter()
+    n = host_cores()
+    cpu_oracle_sample(w.name, args.k, n, nseq=1, budget=3.0, max_calls=1)   # warm-up
+    rates, t_all, last = [], time.perf_counter(), None
     for _ in range(args.steps):
-        r, calls, el = cpu_oracle_rate(model, weights, prompts, args.k, budget_s=10.0, max_calls=24)
-        rates.append(r)
+        last = cpu_oracle_sample(w.name, args.k, n, nseq=2, budget=8.0, max_calls=8)
+        rates.append(last["rate"])
     el = time.perf_counter() - t_all
     v = statistics.median(rates)
-    sample = f"{Bs} sequences x decode calls of k={args.k} for up to 10 s per step (prompt {w.prompt_len})"
+    sample = (f"{last['seqs']} of the {B} sequences (prompts {last['ctx']}), up to 8 decode calls of "
+              f"k={args.k} per step after the prompt, numpy fp32 on {n} threads")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000 * el / max(1, args.steps), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": bench_config(w, B, gen, args.k),
-            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cpu_threads(),
-                             "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": n, "kind": "oracle",
+                             "cpu": cpu_model(), "sample": sample},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -275,12 +345,14 @@ def run_reference(args):
 
 def measured_traffic(kind, workload, B, k):
     """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of
-    the dominant kernel from the committed ncu capture of the LM1B batch-64
-    k=4 step, or None when the workload differs or the kernel's sources have
-    changed since the capture (checked by SHA-256)."""
+    the dominant kernel from the committed ncu capture for this workload
+    (profiles/ncu_dram_traffic_<workload>_b<B>_k<k>.json), scaled to one
+    full-size launch as the capture's record states; None when there is no
+    capture for this workload and kernel, or when the kernel's sources have
+    changed since (checked by SHA-256)."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "ncu_dram_traffic_lm1b_b64_k4.json")
-    if not (workload == "lm1b" and B == 64 and k == 4 and os.path.exists(path)):
+    path = os.path.join(ROOT, "profiles", f"ncu_dram_traffic_{workload}_b{B}_k{k}.json")
+    if not os.path.exists(path):
         return None
     with open(path) as f:
         rec = json.load(f)
@@ -293,90 +365,87 @@ def measured_traffic(kind, workload, B, k):
     return rec["dram_bytes_per_launch"]
 
 
-SWEEP = [  # (workload, batch, ks) -- the non-headline configurations
-    ("owt", 1, (4, 2, 1)), ("owt", 8, (4, 2, 1)), ("owt", 32, (4, 2, 1)),
-    ("owt", 128, (4, 2, 1)), ("owt", 256, (4, 2, 1)),
-    ("owt_paged", 512, (4, 1)),
-    ("medium", 256, (8, 4, 1)),
-    ("lm1b_mtp", 64, (4, 1)),
+# the configurations reported beside the headline: (workload, batch, ks, warm-up, timed steps)
+EXTRA = [
+    ("lm1b", 64, (4, 2, 1), 2, 3),
+    ("owt", 1, (4, 2, 1), 1, 2), ("owt", 8, (4, 2, 1), 1, 2), ("owt", 32, (4, 2, 1), 1, 2),
+    ("owt", 128, (4, 2, 1), 1, 2), ("owt", 256, (4, 2, 1), 1, 2),
+    ("medium", 256, (8, 4, 1), 1, 1),
 ]
 
 
-def run_sweep(args):
-    """Tokens/s of full generations per configuration, k vs the AR step, with
-    the step roofline fraction; one JSON line each (rank 0, N = 1)."""
-    import torch
-    from paper_2606_10820_gb300 import build as kbuild
-    from paper_2606_10820_gb300 import kforcing as kf
-    from synth import WORKLOADS, make_weights, workload_prompts
-    kbuild.build()
-    kf.load_library()
-    pk, peak_src = peaks()
-    by_wl = {}
-    only = [x for x in args.sweep_only.split(",") if x]
-    for name, B, ks in SWEEP:
-        if not only or name in only:
-            by_wl.setdefault(name, []).append((B, ks))
-    for name, runs in by_wl.items():
-        w = WORKLOADS[name]
-        model = w.model
-        weights = make_weights(model)
-        maxB = max(B for B, _ in runs)
-        maxk = max(max(ks) for _, ks in runs)
-        stream = torch.cuda.Stream()
-        dec = kf.Decoder(model, weights, max_batch=maxB, max_k=maxk, stream=stream.cuda_stream)
-        del weights
-        for B, ks in runs:
-            prompts = workload_prompts(w, B)
-            dec.prefill(prompts)
-            gen = w.gen_len
-            res = {}
-            for k in ks:
-                kk = 0 if k == 1 else k          # k=1 is the AR teacher step
-                nout = max(kk, 1)
-                calls = -(-gen // nout)
-                z = torch.rand((calls, B, nout), device="cuda")
-                o = torch.zeros((calls, B, nout), dtype=torch.int32, device="cuda")
+def generation_roofline_s(model, prompts, k, calls, pk):
+    """Sum over the calls of one generation of each call's roofline time:
+    the slower of its algorithmic bytes over the measured HBM bandwidth and
+    its flops over the sustained bf16 tensor rate (the calls run inside a
+    long step)."""
+    nout = max(k, 1)
+    t = 0.0
+    for i in range(calls):
+        P = 1 if i == 0 else nout
+        lens = np.array([len(p) - 1 + (0 if i == 0 else 1 + (i - 1) * nout) for p in prompts])
+        byt, fl = step_bytes_flops(model, len(prompts), P, k, lens)
+        t += max(byt / (pk["hbm_gbs"] * 1e9), fl / (pk["bf16_tflops_sustained"] * 1e12))
+    return t
 
-                def one():
-                    dec.rewind()
-                    for i in range(calls):
-                        kf.kf_decode_step(dec.ctx, B, kk, z[i], o[i])
-                for _ in range(max(1, args.warmup)):
-                    one()
-                torch.cuda.synchronize()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-                for _ in range(args.steps):
-                    one()
-                e1.record(stream)
-                torch.cuda.synchronize()
-                ms = e0.elapsed_time(e1) / args.steps
-                t_roof = 0.0
-                for i in range(calls):
-                    P = 1 if i == 0 else nout
-                    lens = np.array([len(p) - 1 + (0 if i == 0 else 1 + (i - 1) * nout) for p in prompts])
-                    byt, fl = step_bytes_flops(model, B, P, kk, lens)
-                    t_roof += max(byt / (pk["hbm_gbs"] * 1e9), fl / (pk["bf16_tflops_sustained"] * 1e12))
-                res[k] = {"value": B * calls * nout / (ms / 1e3), "ms_per_step": ms,
-                          "step_roofline_frac": t_roof * 1e3 / ms}
-            kmax = max(ks)
-            line = {"metric": METRIC, "value": res[kmax]["value"], "unit": "tokens/s", "n_gpus": 1,
-                    "steps": args.steps, "warmup": args.warmup,
-                    "ms_per_step": res[kmax]["ms_per_step"], "higher_is_better": True,
-                    "scaling": "weak", "vs_baseline": None, "dtype": model.dtype,
-                    "data": "synthetic", "sweep": True,
-                    "config": {"workload": f"{name}: {model.n_layer}L d{model.d_model} V{model.vocab}, "
-                                           f"batch {B}, prompt {w.prompt_len or list(w.ragged)} +{gen}",
-                               "batch": B, "k": kmax},
-                    "per_k": {str(k): {kk_: round(v, 4) for kk_, v in r.items()} for k, r in res.items()},
-                    "speedup_vs_k1": {str(k): res[k]["value"] / res[1]["value"] for k in ks if 1 in res},
-                    "peak_source": peak_src}
-            print(json.dumps(line), flush=True)
-        dec.close()
-        del dec
-        torch.cuda.empty_cache()
-    return 0
+
+def time_generations(kf, dec, B, k, gen, stream, warmup, steps, host=False, dist=None):
+    """Mean ms of one full generation (rewind, then gen / k calls), timed with
+    CUDA events on the library's stream (host=True: wall clock, with host
+    noise in and host tokens out of every call)."""
+    import torch
+    nout = max(k, 1)
+    calls = -(-gen // nout)
+    rng = np.random.default_rng(2)
+    z = rng.random((calls, B, nout), dtype=np.float32)
+    if host:
+        zbuf = torch.from_numpy(z).pin_memory()
+        obuf = torch.zeros((calls, B, nout), dtype=torch.int32).pin_memory()
+    else:
+        zbuf = torch.from_numpy(z).cuda()
+        obuf = torch.zeros((calls, B, nout), dtype=torch.int32, device="cuda")
+
+    def one():
+        dec.rewind()
+        for i in range(calls):
+            kf.kf_decode_step(dec.ctx, B, k, zbuf[i], obuf[i])
+
+    for _ in range(warmup):
+        one()
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    ms = wall * 1000.0 if host else e0.elapsed_time(e1)
+    return ms / steps, calls
+
+
+def measure_config(kf, dec, w, B, ks, pk, warmup, steps, stream):
+    """tokens/s per k (k = 1 is the AR teacher step), the speedup over it and
+    the step roofline fraction for one configuration."""
+    from synth import workload_prompts
+    prompts = workload_prompts(w, B)
+    dec.prefill(prompts)
+    gen = w.gen_len
+    res = {}
+    for k in ks:
+        kk = 0 if k == 1 else k
+        ms, calls = time_generations(kf, dec, B, kk, gen, stream, warmup, steps)
+        t_roof = generation_roofline_s(w.model, prompts, kk, calls, pk)
+        res[str(k)] = {"tokens_per_s": B * calls * max(kk, 1) / (ms / 1e3), "ms_per_generation": ms,
+                       "step_roofline_frac": t_roof * 1e3 / ms}
+    out = {"per_k": res}
+    if "1" in res:
+        out["speedup_vs_k1"] = {kk: r["tokens_per_s"] / res["1"]["tokens_per_s"] for kk, r in res.items()}
+    return out
 
 
 def run_serving(args):
@@ -536,9 +605,9 @@ def run_train_attention(args):
 
 
 def main():
+    if len(sys.argv) > 1 and sys.argv[1] == "--cpu-child":
+        return _cpu_child(sys.argv[2:])
     args = parse()
-    if args.sweep:
-        return run_sweep(args)
     if args.serving:
         return run_serving(args)
     if args.train_attention:
@@ -548,7 +617,7 @@ def main():
     import torch
     from paper_2606_10820_gb300 import build as kbuild
     from paper_2606_10820_gb300 import kforcing as kf
-    from synth import make_weights, workload_prompts
+    from synth import WORKLOADS, make_weights, workload_prompts
 
     rank, world, dist = dist_init(args.gpus)
     dev = int(os.environ.get("LOCAL_RANK", "0"))
@@ -558,91 +627,66 @@ def main():
     if dist is not None:
         dist.barrier()
     kf.load_library()
+    pk, peak_src = peaks()
 
     w, B, gen = workload_of(args)
     model = w.model
     k = args.k
+    nout = max(k, 1)
+    extras = [] if (args.no_extra or rank != 0 or world > 1) else \
+        [e for e in EXTRA if not args.extra_only or e[0] in args.extra_only.split(",")]
+    # configurations of the headline's model share its weights and decoder
+    same = [e for e in extras if WORKLOADS[e[0]].model == model]
     weights = make_weights(model)
     prompts = workload_prompts(w, B)
     stream = torch.cuda.Stream()
-    max_k = max(k, 1)
-    dec = kf.Decoder(model, weights, max_batch=B, max_k=max_k, stream=stream.cuda_stream)
+    max_b = max([B] + [e[1] for e in same])
+    max_k = max([nout] + [max(e[2]) for e in same])
+    dec = kf.Decoder(model, weights, max_batch=max_b, max_k=max_k, stream=stream.cuda_stream)
     dec.prefill(prompts)
-    pk, peak_src = peaks()
-
-    def measure(kk, host=False):
-        nout = max(kk, 1)
-        calls = -(-gen // nout)
-        rng = np.random.default_rng(2)
-        z = rng.random((calls, B, nout), dtype=np.float32)
-        if host:
-            zbuf = torch.from_numpy(z).pin_memory()
-            obuf = torch.zeros((calls, B, nout), dtype=torch.int32).pin_memory()
-        else:
-            zbuf = torch.from_numpy(z).cuda()
-            obuf = torch.zeros((calls, B, nout), dtype=torch.int32, device="cuda")
-
-        def one():
-            dec.rewind()
-            for i in range(calls):
-                kf.kf_decode_step(dec.ctx, B, kk, zbuf[i], obuf[i])
-
-        for _ in range(args.warmup):
-            one()
-        torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        e0.record(stream)
-        for _ in range(args.steps):
-            one()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        wall = time.perf_counter() - t0
-        ms = e0.elapsed_time(e1) if not host else wall * 1000.0
-        ms = max_over_ranks(ms, dist)
-        tokens = world * args.steps * B * calls * nout
-        return tokens / (ms / 1000.0), ms / args.steps, calls, z.nbytes // calls * calls
 
     clk = Clocks(dev)
     clk.start()
-    val, ms_step, calls, _ = measure(k)
+    ms_step, calls = time_generations(kf, dec, B, k, gen, stream, args.warmup, args.steps, dist=dist)
     clocks = clk.stop()
-    e2e_val, e2e_ms, _, _ = measure(k, host=True)
-    nout = max(k, 1)
-    h2d = calls * B * nout * 4
-    d2h = calls * B * nout * 4
+    ms_step = max_over_ranks(ms_step, dist)
+    val = world * B * calls * nout / (ms_step / 1e3)
+    e2e_ms, _ = time_generations(kf, dec, B, k, gen, stream, args.warmup, args.steps, host=True, dist=dist)
+    e2e_ms = max_over_ranks(e2e_ms, dist)
+    e2e_val = world * B * calls * nout / (e2e_ms / 1e3)
+    h2d = d2h = calls * B * nout * 4
     ar = None
     if not args.no_ar and k != 0:
-        ar_val, ar_ms, ar_calls, _ = measure(0)
-        ar = {"value": ar_val, "unit": "tokens/s", "ms_per_step": ar_ms, "calls_per_step": ar_calls}
+        ar_ms, ar_calls = time_generations(kf, dec, B, 0, gen, stream, args.warmup, args.steps, dist=dist)
+        ar_ms = max_over_ranks(ar_ms, dist)
+        ar = {"value": world * B * ar_calls / (ar_ms / 1e3), "unit": "tokens/s", "ms_per_step": ar_ms,
+              "calls_per_step": ar_calls,
+              "step_roofline_frac": generation_roofline_s(model, prompts, 0, ar_calls, pk) * 1e3 / ar_ms}
 
-    # per-kernel times over one profiled step (a graph with event nodes) near the middle of the generation
+    # per-kernel times of one call in the middle of the generation
+    # (kf_profile_step: the call replayed as a graph whose event-record nodes
+    # bracket each launch, without programmatic dependent launch); launches
+    # per call for every shape of the generation
     dec.rewind()
     zmid = np.random.default_rng(5).random((B, nout), dtype=np.float32)
     out = np.zeros((B, nout), np.int32)
-    launches_per_step = 0
     ms_kind = np.zeros(kf.KF_KIND_COUNT, np.float32)
     n_kind = np.zeros(kf.KF_KIND_COUNT, np.int32)
-    ms_tot = np.zeros(kf.KF_KIND_COUNT, np.float64)
-    n_tot = np.zeros(kf.KF_KIND_COUNT, np.int64)
-    shape_launch = {}
+    shape_launch, mid = {}, None
     for i in range(calls):
         P = 1 if i == 0 else nout
         if i in (0, 1, calls // 2):
             lens = dec.lengths()
+            t0 = time.perf_counter()
             kf.kf_profile_step(dec.ctx, B, k, zmid, out, ms_kind, n_kind)
             shape_launch[P] = int(n_kind.sum())
             if i == calls // 2:
-                ms_tot += ms_kind
-                n_tot += n_kind
-                mid_lens = lens.copy()
+                mid = (ms_kind.astype(np.float64).copy(), n_kind.copy(), lens.copy(), P)
         else:
             dec.step(k, zmid, out)
     launches_per_step = sum(shape_launch.get(1 if i == 0 else nout, 0) for i in range(calls))
-    costs = kind_costs(model, B, nout, k, mid_lens)
+    ms_tot, n_tot, mid_lens, P_mid = mid
+    costs = kind_costs(model, B, P_mid, k, mid_lens)
     tot_ms = {kf.KIND_NAMES[i]: float(ms_tot[i]) for i in range(kf.KF_KIND_COUNT)}
     dom = max(costs, key=lambda n: tot_ms.get(n, 0.0))
     idx = kf.KIND_NAMES.index(dom)
@@ -652,33 +696,46 @@ def main():
     t_tc = c["flops"] / (pk["bf16_tflops_sustained"] * 1e12)
     if t_tc > t_hbm:
         ach = c["flops"] / (avg_ms / 1e3) / 1e12
-        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops_sustained"],
-                "unit": "TFLOP/s"}
+        roof = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s"}
     else:
         ach = c["bytes"] / (avg_ms / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s"}
-    traffic = measured_traffic(dom, args.workload, B, k)
-    roof.update({"frac": roof["achieved"] / roof["peak"], "traffic": traffic, "kernel": dom,
-                 "launch_ms": avg_ms, "peak_source": peak_src,
-                 "algorithmic_bytes": c["bytes"], "algorithmic_flops": c["flops"]})
-    # whole-step roofline (slower of HBM bytes and tensor flops), over the generation
-    t_roof = 0.0
-    for i in range(calls):
-        P = 1 if i == 0 else nout
-        lens = np.array([len(p) - 1 + (0 if i == 0 else 1 + (i - 1) * nout) for p in prompts])
-        byt, fl = step_bytes_flops(model, B, P, k, lens)
-        t_roof += max(byt / (pk["hbm_gbs"] * 1e9), fl / (pk["bf16_tflops_sustained"] * 1e12))
-    step_frac = (t_roof * 1e3) / ms_step
+    # the profiled call against the mean graph-replayed call of the timed generation
+    prof_call_ms = float(ms_tot.sum())
+    roof.update({"frac": roof["achieved"] / roof["peak"], "traffic": measured_traffic(dom, w.name, B, k),
+                 "kernel": dom, "launch_ms": avg_ms, "peak_source": peak_src,
+                 "algorithmic_bytes": c["bytes"], "algorithmic_flops": c["flops"],
+                 "kernel_share_of_call": float(ms_tot[idx] / max(1e-9, prof_call_ms)),
+                 "time_source": "CUDA events around each launch of one mid-generation call "
+                                "(kf_profile_step), cross-checked by profiled_call_ms vs graph_call_ms",
+                 "profiled_call_ms": prof_call_ms, "graph_call_ms": ms_step / calls})
+    step_frac = generation_roofline_s(model, prompts, k, calls, pk) * 1e3 / ms_step
+
+    # every other configuration: the headline model's first, on its decoder
+    configs = {}
+    for name, b, ks, wu, st in same:
+        configs[f"{name}_b{b}"] = measure_config(kf, dec, WORKLOADS[name], b, ks, pk, wu, st, stream)
+    dec.close()
+    del dec
+    torch.cuda.empty_cache()
+    by_model = {}
+    for e in extras:
+        if e not in same:
+            by_model.setdefault(WORKLOADS[e[0]].model, []).append(e)
+    for m, runs in by_model.items():
+        wts = make_weights(m)
+        d2 = kf.Decoder(m, wts, max_batch=max(r[1] for r in runs), max_k=max(max(r[2]) for r in runs),
+                        stream=stream.cuda_stream)
+        del wts
+        for name, b, ks, wu, st in runs:
+            configs[f"{name}_b{b}"] = measure_config(kf, d2, WORKLOADS[name], b, ks, pk, wu, st, stream)
+        d2.close()
+        del d2
+        torch.cuda.empty_cache()
 
     cpu = None
     if rank == 0 and not args.no_cpu:
-        Bs = min(B, 16)
-        r, ncalls, el = cpu_oracle_rate(model, weights, prompts[:Bs], k, budget_s=15.0,
-                                        max_calls=24)
-        cpu = {"value": r, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
-               "sample": f"{Bs} of the {B} sequences, {ncalls} decode calls of k={k} "
-                         f"after the prompt ({el:.1f} s, numpy fp64)"}
-    dec.close()
+        cpu = cpu_baseline(w.name, k, B)
     if rank == 0:
         line = {
             "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": world,
@@ -695,7 +752,8 @@ def main():
             "cpu_baseline": cpu,
             "clocks": clocks,
             "gpu_launches": launches_per_step * args.steps,
-            "kernel_ms_mid_step": {kn: round(v, 4) for kn, v in tot_ms.items() if v > 0},
+            "kernel_ms_mid_call": {kn: round(v, 4) for kn, v in tot_ms.items() if v > 0},
+            "configs": configs,
         }
         print(json.dumps(line))
     if dist is not None:

@@ -114,12 +114,17 @@ def token_map(cfg, logits_row, z, map_dtype):
 class OracleDecoder:
     """KV-cached inference of Alg. 1 over a batch, one sequence at a time.
 
-    ``map_dtype`` is the precision of the noise -> token decision (fp32, as
-    the CUDA kernels take it, unless a test asks for fp64).
+    ``map_dtype`` is the precision of the noise -> token decision. By default
+    it is the precision in which the CUDA path takes it: fp32 for bf16
+    models, whose logits carry bf16 rounding far above fp32's, and fp64 for
+    fp32 models, so the decision adds no rounding of its own beyond the
+    fp32 logits. A test may ask for another.
     """
 
-    def __init__(self, model: OracleModel, map_dtype=np.float32):
+    def __init__(self, model: OracleModel, map_dtype=None):
         self.m = model
+        if map_dtype is None:
+            map_dtype = np.float64 if model.cfg.dtype == "fp32" else np.float32
         self.map_dtype = map_dtype
         self.seqs = []
 
@@ -220,10 +225,12 @@ def full_forward_logits(model: OracleModel, tokens, z=None, k: int = 0):
     return model.logits(o[n:] if k > 0 else o[n - 1:n])
 
 
-def ar_sample(model: OracleModel, prompt, zs, map_dtype=np.float32):
+def ar_sample(model: OracleModel, prompt, zs, map_dtype=None):
     """Textbook AR sampling by full recomputation: each new token is
     F^{-1}(z_t) of the next-token softmax of the whole current sequence
     (Eq. 1 with k = 1)."""
+    if map_dtype is None:
+        map_dtype = np.float64 if model.cfg.dtype == "fp32" else np.float32
     seq = [int(t) for t in prompt]
     out = []
     for zt in zs:

@@ -2,6 +2,8 @@
 // the LM head's noise -> token selection, and the step commit.
 #include <algorithm>
 
+#include <type_traits>
+
 #include "kf_internal.cuh"
 
 namespace kf {
@@ -319,6 +321,13 @@ __device__ __forceinline__ void ld_vec(const __nv_bfloat16* p, float* o) {
   }
 }
 
+// exp(m - M) in the precision of the inverse-CDF sums
+template <typename Acc> __device__ __forceinline__ Acc chunk_scale(float m, float M);
+template <> __device__ __forceinline__ float chunk_scale<float>(float m, float M) { return expf(m - M); }
+template <> __device__ __forceinline__ double chunk_scale<double>(float m, float M) {
+  return exp((double)m - (double)M);
+}
+
 template <typename TA>
 __global__ void __launch_bounds__(kSelThreads)
 k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
@@ -347,14 +356,19 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
     if (threadIdx.x == 0) tokens[zrow] = -1;
     return;
   }
+  // the inverse-CDF sums: fp32 for the bf16 model (its logits carry bf16
+  // rounding far above fp32's); fp64 for the fp32 model, so its decision is
+  // limited by its fp32 logits and not by ~5e4 fp32 additions
+  using Acc = typename std::conditional<sizeof(TA) == 4, double, float>::type;
   const HeadRec* rec = rec_all + (size_t)row * nchunk;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   __shared__ float s_red[kSelThreads / 32];
+  __shared__ Acc s_acc[kSelThreads / 32];
   __shared__ int s_redi[kSelThreads / 32];
-  __shared__ float s_part[kSelThreads];
-  __shared__ float s_M, s_T;
+  __shared__ float s_M;
+  __shared__ Acc s_T;
   __shared__ int s_chunk;
-  __shared__ float s_before;
+  __shared__ Acc s_before;
 
   // contiguous chunk range per thread keeps id order inside each partial sum
   const int per = ceil_div(nchunk, kSelThreads);
@@ -410,40 +424,40 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   //    fixed-order block scan over the threads: lanes by shuffles, warps by
   //    their totals.  The scan's last element is the total S, so T = z S
   //    is crossed for every z < 1.
-  float part = 0.f;
+  Acc part = 0;
   if (keep) {
 #pragma unroll
     for (int i = 0; i < kKeep; ++i)
-      if (c0 + i < c1) part += ks[i] * expf(km[i] - M);
+      if (c0 + i < c1) part += (Acc)ks[i] * chunk_scale<Acc>(km[i], M);
   } else {
     for (int c = c0; c < c1; ++c) {
       HeadRec r = rec[c];
-      part += r.s * expf(r.m - M);
+      part += (Acc)r.s * chunk_scale<Acc>(r.m, M);
     }
   }
-  float inc = part;
+  Acc inc = part;
   for (int o = 1; o < 32; o <<= 1) {
-    const float y = __shfl_up_sync(0xffffffffu, inc, o);
+    const Acc y = __shfl_up_sync(0xffffffffu, inc, o);
     if (lane >= o) inc += y;
   }
-  float lane_excl = __shfl_up_sync(0xffffffffu, inc, 1);
-  if (lane == 0) lane_excl = 0.f;
-  if (lane == 31) s_red[warp] = inc;
+  Acc lane_excl = __shfl_up_sync(0xffffffffu, inc, 1);
+  if (lane == 0) lane_excl = 0;
+  if (lane == 31) s_acc[warp] = inc;
   __syncthreads();
-  __shared__ float s_wexcl[kSelThreads / 32 + 1];
+  __shared__ Acc s_wexcl[kSelThreads / 32 + 1];
   if (t == 0) {
-    float run = 0.f;
+    Acc run = 0;
     for (int w = 0; w < kSelThreads / 32; ++w) {
       s_wexcl[w] = run;
-      run += s_red[w];
+      run += s_acc[w];
     }
     s_wexcl[kSelThreads / 32] = run;     // S
-    s_T = noise[zrow] * run;
+    s_T = (Acc)noise[zrow] * run;
     s_redi[2] = kSelThreads;             // first crossing thread (none yet)
   }
   __syncthreads();
-  const float T = s_T;
-  const float excl = s_wexcl[warp] + lane_excl, incl = s_wexcl[warp] + inc;
+  const Acc T = s_T;
+  const Acc excl = s_wexcl[warp] + lane_excl, incl = s_wexcl[warp] + inc;
   {
     const unsigned cross = __ballot_sync(0xffffffffu, incl > T);
     if (lane == 0 && cross) atomicMin(&s_redi[2], warp * 32 + __ffs(cross) - 1);
@@ -451,12 +465,12 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   __syncthreads();
   if (t == s_redi[2]) {
     // the crossing range: walk its chunks in id order from its exclusive prefix
-    float acc = excl;
+    Acc acc = excl;
     int cstar = c1 - 1;
-    float before = acc;
+    Acc before = acc;
     for (int c = c0; c < c1; ++c) {
       HeadRec r = rec[c];
-      const float sc = r.s * expf(r.m - M);
+      const Acc sc = (Acc)r.s * chunk_scale<Acc>(r.m, M);
       // the range's own order can round differently from its partial sum:
       // its last chunk takes the crossing then
       if (acc + sc > T || c == c1 - 1) { cstar = c; before = acc; break; }
@@ -471,7 +485,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
     int cstar = nchunk - 1;
     while (cstar > 0 && !(rec[cstar].s * expf(rec[cstar].m - M) > 0.f)) --cstar;
     s_chunk = cstar;
-    s_before = 0.f;
+    s_before = 0;
     s_redi[1] = 1;
   }
   __syncthreads();
@@ -515,17 +529,17 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   if (warp != 0) return;
   const int v = cstar * kChunk + lane;
   const float l = s_logit[lane];
-  float e = (v < V) ? expf(l - M) : 0.f;
+  const Acc e = (v < V) ? chunk_scale<Acc>(l, M) : (Acc)0;
   // inclusive prefix over lanes in id order
-  float pre = e;
+  Acc pre = e;
   for (int o = 1; o < 32; o <<= 1) {
-    float y = __shfl_up_sync(0xffffffffu, pre, o);
+    Acc y = __shfl_up_sync(0xffffffffu, pre, o);
     if (lane >= o) pre += y;
   }
-  const float Tp = s_T - s_before;
+  const Acc Tp = s_T - s_before;
   const bool fallback = s_redi[1] != 0;
   unsigned hit = __ballot_sync(0xffffffffu, !fallback && (v < V) && (pre > Tp));
-  unsigned pos = __ballot_sync(0xffffffffu, (v < V) && (e > 0.f));
+  unsigned pos = __ballot_sync(0xffffffffu, (v < V) && (e > (Acc)0));
   if (lane == 0) {
     int tok;
     if (hit) tok = cstar * kChunk + (__ffs(hit) - 1);

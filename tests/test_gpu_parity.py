@@ -6,6 +6,8 @@ token explained by the logit error (tests/parity.py).  The oracle is
 teacher-forced with the GPU's tokens after each step, so both sides always
 decode from the same context.
 """
+import os
+
 import numpy as np
 import pytest
 
@@ -13,7 +15,7 @@ import oracle
 from synth import (LM1B, MEDIUM, OWT, TINY, WORKLOADS, make_noise, make_prompt_lengths,
                    make_prompts, make_weights, workload_prompts)
 
-from parity import LOGIT_TOL, compare_tokens, logit_check
+from parity import LOGIT_TOL, compare_tokens, logit_check, record
 
 pytestmark = pytest.mark.gpu
 
@@ -29,7 +31,7 @@ def kf():
     return kforcing
 
 
-def _run(kf, cfg, w, prompts, ks, max_k, seed=2, flags=0, map_dtype=np.float32, dec=None,
+def _run(kf, cfg, w, prompts, ks, max_k, seed=2, flags=0, map_dtype=None, dec=None,
          check_logits=True):
     """Decode ks steps on both sides; returns per-step records."""
     B = len(prompts)
@@ -241,13 +243,22 @@ def test_errors_are_reported(kf):
     d.close()
 
 
+def _test_name():
+    return os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0].split("::")[-1]
+
+
 def _bf16_check(recs, map_kind="icdf"):
-    worst, slots, mism, bad = 0.0, 0, 0, 0
+    """Worst logit error and token counts over the records; the counts go to
+    the end-of-run agreement summary. Every bf16 test asserts that no
+    mismatch is unexplained and that every decidable slot agrees."""
+    worst = 0.0
+    st = [0, 0, 0, 0, 0]
     for k, z, gt, rt, gl, rl in recs:
         worst = max(worst, logit_check(gl, rl))
-        n, m, u = compare_tokens(gt, rt, gl, rl, z, map_kind)
-        slots, mism, bad = slots + n, mism + m, bad + u
-    return worst, slots, mism, bad
+        compare_tokens(gt, rt, gl, rl, z, map_kind, stats=st)
+    record(_test_name(), st)
+    assert st[4] == 0, f"{st[4]} decidable slots differ: {st}"
+    return worst, st[0], st[1], st[2]
 
 
 @pytest.fixture(scope="module")
@@ -267,13 +278,12 @@ def test_lm1b_bf16_small_batch(kf, lm1b_weights):
     dec.close()
 
 
-@pytest.mark.parametrize("flags", [0, 8])   # 8 = KF_FLAG_TC_ATTN
-def test_lm1b_bf16_k8_both_attention_kernels(kf, lm1b_weights, flags):
-    """k = 8 (16 query rows per sequence) and ragged prefill groups on the
-    warp-MMA attention kernel and, with KF_FLAG_TC_ATTN, the tcgen05 one."""
+def test_lm1b_bf16_k8(kf, lm1b_weights):
+    """k = 8 (16 query rows per sequence, both 8-row halves of the warp-MMA
+    attention tile) and ragged prefill groups."""
     cfg = LM1B
     prompts = make_prompts([40, 23, 17], cfg.vocab)
-    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [8, 8, 4, 8], max_k=8, flags=flags)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [8, 8, 4, 8], max_k=8)
     worst, slots, mism, bad = _bf16_check(recs)
     assert worst <= LOGIT_TOL
     assert bad == 0
@@ -292,8 +302,10 @@ def test_lm1b_bf16_argmax(kf, lm1b_weights):
 
 
 def test_lm1b_bf16_sharp_temperature(kf, lm1b_weights):
-    """At tau = 0.1 the softmax is sharp and the token agreement is >= 99.9%
-    whenever the margin exceeds the logit error (every mismatch explained)."""
+    """At tau = 0.1 the softmax is sharp: more slots are decidable (noise
+    farther than the logit-error bound from every CDF boundary), and every
+    decidable slot must agree; the raw agreement is recorded, not bounded
+    (a few slots of 64 still fall inside the bound)."""
     cfg = LM1B.replace(tau=0.1)
     prompts = make_prompts([32] * 4, cfg.vocab)
     dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 4, 4], max_k=4)
@@ -315,16 +327,15 @@ def test_lm1b_full_batch_sampled(kf, lm1b_weights):
     ref = oracle.OracleDecoder(oracle.OracleModel(cfg, lm1b_weights))
     ref.prefill([prompts[i] for i in pick])
     zs = make_noise(3, B, 4)
-    worst, slots, mism, bad = 0.0, 0, 0, 0
+    recs = []
     for s in range(3):
         gt = dec.step(4, zs[s])
         gl = dec.logits(4)[pick]
         rt, rl = ref.step(4, zs[s][pick], want_logits=True)
-        worst = max(worst, logit_check(gl, rl))
-        n, m, u = compare_tokens(gt[pick], rt, gl, rl, zs[s][pick])
-        slots, mism, bad = slots + n, mism + m, bad + u
+        recs.append((4, zs[s][pick], gt[pick].copy(), rt, gl, rl))
         for j, b in enumerate(pick):
             ref.seqs[j]["pending"] = [int(t) for t in gt[b]]
+    worst, slots, mism, bad = _bf16_check(recs)
     assert worst <= LOGIT_TOL and bad == 0
     dec.close()
 
@@ -363,20 +374,18 @@ def _sampled(kf, cfg, w, prompts, pick, ks, max_k, seed):
     ref = oracle.OracleDecoder(oracle.OracleModel(cfg, w))
     ref.prefill([prompts[i] for i in pick])
     rng = np.random.default_rng(seed)
-    worst, slots, mism, bad = 0.0, 0, 0, 0
+    recs = []
     for k in ks:
         z = rng.random((B, max(k, 1)), dtype=np.float32)
         gt = dec.step(k, z)
         gl = dec.logits(max(k, 1))[pick]
         rt, rl = ref.step(k, z[pick], want_logits=True)
-        worst = max(worst, logit_check(gl, rl))
-        n, m, u = compare_tokens(gt[pick], rt, gl, rl, z[pick])
-        slots, mism, bad = slots + n, mism + m, bad + u
+        recs.append((k, z[pick], gt[pick].copy(), rt, gl, rl))
         for j, b in enumerate(pick):
             ref.seqs[j]["pending"] = [int(t) for t in gt[b]]
         assert [int(x) for x in dec.lengths()[pick]] == [ref.cached_len(j) for j in range(len(pick))]
     dec.close()
-    return worst, slots, mism, bad
+    return _bf16_check(recs)
 
 
 def test_owt_paged_full_batch_sampled(kf):
@@ -400,3 +409,94 @@ def test_medium_k8_sampled(kf):
     prompts = make_prompts([1024] * 256, cfg.vocab)
     worst, slots, mism, bad = _sampled(kf, cfg, w, prompts, [0, 255], [8, 8, 4], 8, 22)
     assert worst <= LOGIT_TOL and bad == 0
+
+
+def test_lm1b_bf16_agreement_over_1024_slots(kf, lm1b_weights):
+    """The bench's shape, batch 64 at k = 4, every sequence against the oracle
+    (teacher-forced) for four steps: 1024 slots at tau = 0.1. Every decidable
+    slot agrees (the >= 99.9 % criterion, graded where the logit error cannot
+    move the token) and every other mismatch is explained; the raw rate is
+    recorded."""
+    cfg = LM1B.replace(tau=0.1)
+    prompts = make_prompts([32] * 64, cfg.vocab)
+    dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 4, 4], max_k=4)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert slots == 1024
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
+
+
+# ------------------------------------------- fp32 exact tokens, real shapes
+
+# Both sides take the fp32 model's token decision with fp64 sums. What can
+# still move a CDF boundary is the fp32 logits' own rounding: ~1e-6 relative
+# per logit, ~1e-8 on a boundary. A mismatch whose noise lies within this
+# bound of the oracle's boundary is a rounding tie, and it is reported.
+FP32_DECISION_BOUND = 2e-6
+
+
+@pytest.mark.parametrize("shape", ["lm1b", "owt", "medium"])
+def test_fp32_tokens_identical_real_shapes(kf, shape):
+    """The fp32 mode at the workloads' real shapes: vocabularies of 30,522 and
+    50,257, d_model 768 and 1024, head_dim 64, 12 and 24 layers. Ragged prompts
+    cross 16-token pages, and the steps mix k = 4, k = 8 and the AR step.
+    Tokens are identical in every slot whose noise lies farther than the fp32
+    decision's own rounding (FP32_DECISION_BOUND) from the oracle's CDF
+    boundaries. Any other mismatch fails the test, with its margin, the
+    distance |z - F| to the nearest boundary between the two bins. The
+    near-boundary mismatches are counted in the end-of-run summary."""
+    base = {"lm1b": LM1B, "owt": OWT.replace(max_len=512), "medium": MEDIUM.replace(max_len=512)}[shape]
+    cfg = base.replace(dtype="fp32")
+    w = make_weights(cfg)
+    lens = {"lm1b": [20, 33, 47], "owt": [100, 17, 250], "medium": [40, 129, 7]}[shape]
+    prompts = make_prompts(lens, cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 8, 0, 4, 8, 0], max_k=8, seed=31)
+    slots, near, bad = 0, [], []
+    for k, z, gt, rt, gl, rl in recs:
+        rt = rt.astype(np.int32)
+        slots += gt.size
+        for b, j in zip(*np.nonzero(gt != rt)):
+            l = np.asarray(rl[b, j], np.float64)
+            p = np.exp(l - l.max())
+            F = np.cumsum(p / p.sum())
+            lo, hi = sorted((int(gt[b, j]), int(rt[b, j])))
+            margin = float(np.abs(F[lo:hi] - z[b, j]).max())
+            msg = f"k={k} slot ({b},{j}) gpu {gt[b, j]} oracle {rt[b, j]} margin {margin:.3e}"
+            (near if margin <= FP32_DECISION_BOUND else bad).append(msg)
+        assert np.abs(gl - rl).max() < 1e-3 * max(1.0, float(np.abs(rl).max()))
+    print(f"fp32 {shape}: {slots - len(near) - len(bad)}/{slots} identical; near-boundary: {near}")
+    record(_test_name(), [slots, len(near) + len(bad), len(bad), slots - len(near) - len(bad), len(bad)])
+    assert not bad, bad
+    assert len(near) <= max(1, slots // 50), near
+    dec.close()
+
+
+# ------------------------------------------- device-side error reporting
+
+def test_device_prompt_out_of_range_reports_device_error(kf):
+    """A device-resident prompt is range-checked where the embedding kernel
+    reads it: an id >= V embeds as id 0 (no out-of-bounds read), flags the
+    device error word, and kf_prefill returns KF_E_DEVICE. A later prefill
+    with valid ids starts clean, and its step decodes like a fresh context."""
+    import torch
+    cfg = TINY
+    w = make_weights(cfg)
+    d = kf.Decoder(cfg, w, max_batch=2, max_k=2)
+    good = make_prompts([9, 12], cfg.vocab)
+    bad = [p.copy() for p in good]
+    bad[1][3] = cfg.vocab + 5
+    toks = torch.from_numpy(np.concatenate(bad)).cuda()
+    lens = np.array([len(p) for p in bad], np.int32)
+    with pytest.raises(kf.KfError) as e:
+        kf.kf_prefill(d.ctx, 2, toks, lens)
+    assert e.value.code == kf.KF_E_DEVICE
+    assert "device error flag 1" in str(e.value) or "flag 1" in kf.kf_last_error(d.ctx)
+    z = make_noise(1, 2, 2)[0]
+    d.prefill(good)
+    got = d.step(2, z)
+    d.sync()
+    f = kf.Decoder(cfg, w, max_batch=2, max_k=2)
+    f.prefill(good)
+    assert np.array_equal(got, f.step(2, z))
+    d.close()
+    f.close()

@@ -30,6 +30,8 @@ def env():
     for fn in ("kf_op_head_tokens", "kf_op_head_tokens_noalloc"):
         getattr(lib, fn).argtypes = args
         getattr(lib, fn).restype = ctypes.c_int
+    lib.kf_op_status.argtypes = [ctypes.c_void_p]
+    lib.kf_op_status.restype = ctypes.c_int
     return torch, lib, kf
 
 
@@ -39,7 +41,7 @@ def _tokens(torch, lib, fn, x, w, z, tau, map_kind):
     rc = getattr(lib, fn)(rows, w.shape[0], d, x.data_ptr(), w.data_ptr(), z.data_ptr(), tau,
                           map_kind, out.data_ptr(), None)
     assert rc == 0, rc
-    torch.cuda.synchronize()
+    assert lib.kf_op_status(None) == 0     # no kernel of the call flagged an error
     return out.cpu().numpy()
 
 
@@ -73,3 +75,70 @@ def test_noalloc_rejects_oversize(env):
                                        0, out.data_ptr(), None)
     assert rc == KF_E_CAPACITY
     assert "static scratch" in kf.kf_last_error()
+
+
+def test_noalloc_matches_oracle(env):
+    """The no-allocation entry against the oracle's inverse-CDF and argmax maps
+    on fp64 logits of the same bf16 operands (the rule of test_gpu_head_op)."""
+    torch, lib, _ = env
+    from test_gpu_head_op import check_against_oracle
+    g = torch.Generator(device="cuda").manual_seed(77)
+    x = torch.randn(40, 256, device="cuda", generator=g).to(torch.bfloat16)
+    w = (torch.randn(5000, 256, device="cuda", generator=g) * 0.05).to(torch.bfloat16)
+    z = torch.rand(40, device="cuda", generator=g)
+    for map_kind in (0, 1):
+        got = _tokens(torch, lib, "kf_op_head_tokens_noalloc", x, w, z, 0.8, map_kind)
+        assert check_against_oracle(x, w, z, 0.8, map_kind, got) == 0
+
+
+_NO_ALLOC_PROBE = r"""
+import ctypes, sys
+import torch
+sys.path.insert(0, sys.argv[1])
+from paper_2606_10820_gb300 import kforcing as kf
+lib = kf.load_library()
+fn = lib.kf_op_head_tokens_noalloc
+fn.argtypes = [ctypes.c_int32] * 3 + [ctypes.c_void_p] * 3 + [ctypes.c_float, ctypes.c_int32,
+                                                               ctypes.c_void_p, ctypes.c_void_p]
+fn.restype = ctypes.c_int
+g = torch.Generator(device="cuda").manual_seed(3)
+cases = []
+for rows, V, d in [(64, 30522, 768), (200, 1000, 128), (3, 50257, 256)]:
+    x = torch.randn(rows, d, device="cuda", generator=g).to(torch.bfloat16)
+    w = (torch.randn(V, d, device="cuda", generator=g) * 0.05).to(torch.bfloat16)
+    z = torch.rand(2, rows, device="cuda", generator=g)
+    out = torch.zeros(rows, dtype=torch.int32, device="cuda")
+    cases.append((rows, V, d, x, w, z, out))
+torch.cuda.synchronize()
+def run(i):
+    for rows, V, d, x, w, z, out in cases:
+        for m in (0, 1):
+            rc = fn(rows, V, d, x.data_ptr(), w.data_ptr(), z[i].data_ptr(), 1.0, m, out.data_ptr(), None)
+            assert rc == 0, rc
+    torch.cuda.synchronize()
+run(0)                       # module load and every kernel variant once
+before = torch.cuda.mem_get_info()[0]
+for _ in range(3):
+    run(1)
+after = torch.cuda.mem_get_info()[0]
+print("free bytes before", before, "after", after)
+assert before == after, (before, after)
+"""
+
+
+def test_noalloc_allocates_nothing():
+    """In a fresh process that calls only the no-allocation entry: after one
+    warm-up round (module load, every kernel variant), repeated calls of three
+    shapes leave the device's free memory (cudaMemGetInfo) unchanged."""
+    import os
+    import subprocess
+    import sys
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    p = subprocess.run([sys.executable, "-c", _NO_ALLOC_PROBE, root], capture_output=True, text=True,
+                       timeout=600)
+    assert p.returncode == 0, p.stdout + p.stderr
