@@ -51,6 +51,9 @@ struct TcArgs {
   int M, N, K;
   int kb_per_split;   // K blocks per split
   int splits;
+  uint32_t a_box;     // bytes of one A box: its rows (min(128, M rounded up to 8)) x 128
+  const char* l2_next;   // the next projection's weights, prefetched into L2 (or NULL)
+  unsigned long long l2_bytes;
   int* d_err;
   Epi epi;
 };
@@ -125,10 +128,22 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       // stream in while the predecessor kernel finishes; the activation tiles
       // it produces are loaded after pdl_wait.
       const int pre = min(nst, STAGES);
+      if (g.l2_next) {
+        // this CTA's share of the next projection's weights, into L2 for the
+        // kernel after this one (256-byte slices, one prefetch each of at
+        // most 1 MiB)
+        const unsigned long long nct = (unsigned long long)gridDim.x * gridDim.y * gridDim.z;
+        const unsigned long long cta = ((unsigned long long)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+        const unsigned long long per = ((g.l2_bytes + nct - 1) / nct + 255) & ~255ull;
+        for (unsigned long long o = cta * per; o < min(g.l2_bytes, (cta + 1) * per); o += (1u << 20)) {
+          const unsigned long long n = min(min((unsigned long long)(1u << 20), (cta + 1) * per - o), g.l2_bytes - o);
+          prefetch_l2(g.l2_next + o, (uint32_t)(n & ~15ull));
+        }
+      }
       for (int i = 0; i < pre; ++i) {
         const uint32_t full = smem_u32(&bars[i]);
         const int na = min(AT, nkb - i * AT);
-        mbar_expect_tx(full, na * (MT * A_ATOM + B_ATOM));
+        mbar_expect_tx(full, na * (MT * g.a_box + B_ATOM));
         for (int a = 0; a < na; ++a)
           tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES + a * B_ATOM, &map_w, full,
                       (kb0 + i * AT + a) * kBK, n0);
@@ -147,7 +162,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         if (!mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, g.d_err)) break;
         const uint32_t full = smem_u32(&bars[s]);
         const int na = min(AT, nkb - i * AT);
-        mbar_expect_tx(full, na * (MT * A_ATOM + B_ATOM));
+        mbar_expect_tx(full, na * (MT * g.a_box + B_ATOM));
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
         for (int a = 0; a < na; ++a) {
           const int kc = (kb0 + i * AT + a) * kBK;
@@ -332,7 +347,37 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     // over DSMEM, adding the splits in order (deterministic), and runs the
     // epilogue on them.  Every thread of every CTA takes both barriers.
     cluster_sync();
-    if (warp >= 2) {
+    if (EPI == EPI_QKV && warp >= 2) {
+      // QKV: RoPE rotates columns (i, i + 32) of each 64-wide head block, so a
+      // thread takes four columns of the block's first half and the same
+      // four of its second half
+      constexpr int GQ = BN / 8;                   // (block, 4-column group) pairs per row
+      const int S = g.splits;
+      const int q = (int)cluster_rank();
+      const int et = threadIdx.x - 64;
+      const int items = ((kBM - q + S - 1) / S) * GQ;
+      const uint32_t pbase = smem_u32(smem);
+      for (int idx = et; idx < items; idx += 32 * kEpiWarps) {
+        const int rr = q + S * (idx / GQ);
+        const int pr = idx % GQ;
+        const int blk = (pr / 8) * 64, g4 = (pr % 8) * 4;
+        const int row = m0 + rr;
+        if (row >= g.M) continue;
+        float4 lo = make_float4(0.f, 0.f, 0.f, 0.f), hi = lo;
+        const uint32_t off = (uint32_t)((rr * (BN + 4) + blk + g4) * 4);
+        for (int sp = 0; sp < S; ++sp) {
+          const float4 a = ld_dsmem4(pbase + off, (uint32_t)sp);
+          const float4 b = ld_dsmem4(pbase + off + 32 * 4, (uint32_t)sp);
+          lo.x += a.x; lo.y += a.y; lo.z += a.z; lo.w += a.w;
+          hi.x += b.x; hi.y += b.y; hi.z += b.z; hi.w += b.w;
+        }
+        if (g.epi.ss_in) {
+          lo = scale4(lo, meta->rinv[rr]);
+          hi = scale4(hi, meta->rinv[rr]);
+        }
+        epi_qkv<__nv_bfloat16>(g.epi, row, meta->pos[rr], meta->aux[rr], n0 + blk, g4, lo, hi);
+      }
+    } else if (warp >= 2) {
       // this CTA's rows q, q + S, ...: each thread takes U groups of four
       // columns at a time and issues all their DSMEM loads before the
       // epilogue stores, so the latencies overlap
@@ -376,7 +421,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
             }
           }
         }
-        if (EPI != EPI_HEAD && EPI != EPI_QKV) {   // never split (host guarantees)
+        if (EPI != EPI_HEAD && EPI != EPI_QKV) {   // the LM-head records never split; QKV above
 #pragma unroll
           for (int u = 0; u < U; ++u) {
             if (EPI == EPI_BIAS_GELU && ok[u] && g.epi.ss_in) acc[u] = scale4(acc[u], meta->rinv[row[u] - m0]);
@@ -473,8 +518,9 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
   // split K over a cluster of up to 8 CTAs when the tiles alone leave SMs
   // idle: the largest power of two that keeps one wave and two K blocks per
   // split (odd cluster sizes measured slower)
+  // (QKV only within one M tile: at 256 rows its 2-way split measured slower)
   int splits = 1;
-  if (EPI != EPI_HEAD && EPI != EPI_QKV)
+  if (EPI != EPI_HEAD && (EPI != EPI_QKV || m_tiles == 1))
     while (splits < 8 && tiles * splits * 2 <= num_sms && kb_total >= splits * 4) splits *= 2;
   int kbps = ceil_div(kb_total, splits);
   splits = ceil_div(kb_total, kbps);   // no empty splits
@@ -505,11 +551,19 @@ static int launch_epi(const GemmDesc& g, int* d_err, int num_sms, cudaStream_t s
     kbps = ceil_div(kb_total, splits);
     splits = ceil_div(kb_total, kbps);
   }
+  // A boxes cover only the rows a tile can hold: at M <= 128 the 128-row MMA
+  // reads the rows past the box from stale shared memory, and those rows of
+  // the accumulator (all >= M) are never stored
+  const int a_rows = MT == 1 ? std::min(kBM, round_up(g.M, 8)) : kBM;
   CUtensorMap ma, mw;
-  if (!make_map(&ma, g.A, g.M, g.K, g.lda, kBM) || !make_map(&mw, g.W, g.N, g.K, g.ldw, BN))
+  if (!make_map(&ma, g.A, g.M, g.K, g.lda, a_rows) || !make_map(&mw, g.W, g.N, g.K, g.ldw, BN))
     return -1;
   TcArgs a;
   a.M = g.M; a.N = g.N; a.K = g.K; a.kb_per_split = kbps; a.splits = splits;
+  a.a_box = (uint32_t)a_rows * kBK * 2;
+  const bool pf = g.l2_next && g.l2_bytes >= 16 && !(reinterpret_cast<uintptr_t>(g.l2_next) & 15);
+  a.l2_next = pf ? static_cast<const char*>(g.l2_next) : nullptr;
+  a.l2_bytes = pf ? (g.l2_bytes & ~(size_t)15) : 0;
   a.d_err = d_err; a.epi = g.epi;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_tiles, m_tiles, splits);

@@ -402,6 +402,10 @@ struct GemmDesc {
   const void* W;   // [N][ldw] storage TA
   int ldw;
   Epi epi;
+  // weights of the next projection of the step: the tensor-core kernel's CTAs
+  // prefetch them into L2 at their start (16-byte aligned), or NULL
+  const void* l2_next = nullptr;
+  size_t l2_bytes = 0;
 };
 
 // SIMT GEMM (any storage type; fp32 accumulation, k ascending per output)
