@@ -52,6 +52,8 @@ extern "C" {
 #define KF_FLAG_NO_GRAPH 1       /* launch kernels eagerly instead of replaying a CUDA graph */
 #define KF_FLAG_SIMT_GEMM 2      /* bf16 mode: use the SIMT GEMM, not tcgen05   */
 #define KF_FLAG_NO_PDL 4         /* launch without programmatic dependent launch */
+#define KF_FLAG_NO_PERSISTENT_GEMM 16 /* bf16: one CTA per output tile even when the
+                                    tiles exceed a wave (no persistent tile loop) */
 
 /*
  * Model and runtime configuration.  Table 4 gives the backbone (pre-norm

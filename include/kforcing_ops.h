@@ -15,6 +15,8 @@ extern "C" {
 
 #define KF_GEMM_TCGEN05 0   /* tcgen05 + TMEM tensor-core kernel, TMA fed   */
 #define KF_GEMM_SIMT 1      /* CUDA-core kernel, fp32 FMA in ascending k    */
+#define KF_GEMM_TCGEN05_PER_TILE 2 /* the tcgen05 kernel with one CTA per tile
+                                      even past a wave of tiles            */
 
 /*
  * out[M][N] = A[M][K] . W[N][K]^T in fp32: the dense projections of the

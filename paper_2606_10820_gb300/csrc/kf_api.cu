@@ -18,6 +18,7 @@ using namespace kf;
 
 namespace kf {
 thread_local bool g_pdl = false;
+thread_local int g_gemm_flags = 0;
 }
 
 namespace kf {
@@ -199,6 +200,7 @@ static void gemm(kf_ctx* c, int kind, int M, int N, int K, const void* A, int ld
   g.l2_bytes = l2_bytes;
   prof_begin(c, kind);
   bool use_tc = c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && tc_gemm_supported(g);
+  g_gemm_flags = (c->cfg.flags & KF_FLAG_NO_PERSISTENT_GEMM) ? kGemmNoPersist : 0;
   if (use_tc) {
     if (launch_gemm_tc(g, c->d_err, c->stream) != 0) c->launch_failed = true;
   }

@@ -378,6 +378,9 @@ __device__ __forceinline__ void pdl_trigger() {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 extern thread_local bool g_pdl;   // launch with the programmatic-serialization attribute
+// tensor-core GEMM launch options for the launches made by this thread
+constexpr int kGemmNoPersist = 1;  // one CTA per tile even past a wave of tiles
+extern thread_local int g_gemm_flags;
 
 template <typename... KArgs, typename... Args>
 inline void kf_launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,

@@ -74,8 +74,9 @@ extern "C" int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, co
   g.epi.outf = out;
   g.epi.ldo = N;
   cudaStream_t s = (cudaStream_t)stream;
-  if (impl == KF_GEMM_TCGEN05) {
+  if (impl == KF_GEMM_TCGEN05 || impl == KF_GEMM_TCGEN05_PER_TILE) {
     if (!tc_gemm_supported(g)) return KF_E_ARG;
+    g_gemm_flags = impl == KF_GEMM_TCGEN05_PER_TILE ? kGemmNoPersist : 0;
     int dev = 0;
     if (current_device(&dev) != KF_OK) return KF_E_CUDA;
     int* err = nullptr;

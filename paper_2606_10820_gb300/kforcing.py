@@ -22,7 +22,7 @@ KF_OK, KF_E_ARG, KF_E_CAPACITY, KF_E_OOM, KF_E_CUDA, KF_E_DEVICE, KF_E_STATE = 0
 KF_POS_ROPE, KF_POS_LEARNED = 0, 1
 KF_DTYPE_FP32, KF_DTYPE_BF16 = 0, 1
 KF_MAP_ICDF, KF_MAP_ARGMAX = 0, 1
-KF_FLAG_NO_GRAPH, KF_FLAG_SIMT_GEMM, KF_FLAG_NO_PDL = 1, 2, 4
+KF_FLAG_NO_GRAPH, KF_FLAG_SIMT_GEMM, KF_FLAG_NO_PDL, KF_FLAG_NO_PERSISTENT_GEMM = 1, 2, 4, 16
 KIND_NAMES = ["rowmap", "embed", "noise_gemm", "rmsnorm", "gemm_qkv", "rope_kv", "attention",
               "attn_combine", "gemm_o", "gemm_up", "gemm_down", "head_norm", "gemm_head",
               "head_select", "commit"]

@@ -18,9 +18,12 @@ SHAPES = [
     (256, 30720, 768),   # LM-head shape (vocab padded to 256)
     (1000, 200, 128),    # N not a multiple of the tile
     (200, 640, 320),     # odd number of 64-wide K blocks: a short last pipeline stage
-    (4096, 768, 3072),   # large M
-    (2100, 2340, 768),   # 256-wide tiles with ragged M and N
+    (4096, 768, 3072),   # large M: persistent 256-wide tiles
+    (2100, 2340, 768),   # persistent 256-wide tiles with ragged M and N
+    (4096, 2304, 768),   # OWT batch 512 k=4 QKV shape: two tiles per CTA
 ]
+
+PERSISTENT = [(4096, 768, 3072), (2100, 2340, 768), (4096, 2304, 768)]
 
 
 @pytest.fixture(scope="module")
@@ -55,11 +58,22 @@ def test_gemm_matches_fp32_matmul(env, M, N, K):
     W = (torch.randn(N, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
     ref = (A.double() @ W.double().T).float()
     scale = ref.abs().max().item()
-    for impl in (0, 1):
+    for impl in (0, 1, 2):     # tcgen05, SIMT, tcgen05 one CTA per tile
         out = _run(torch, lib, impl, A, W)
         assert torch.isfinite(out).all()
         err = (out - ref).abs().max().item()
         assert err <= 1e-4 * scale + 1e-6, (impl, err, scale)
+
+
+@pytest.mark.parametrize("M,N,K", PERSISTENT)
+def test_persistent_tiles_equal_per_tile_ctas(env, M, N, K):
+    """Past a wave of tiles the persistent tile loop computes each 128 x 256
+    tile with the same K order as a CTA per tile: identical bits."""
+    torch, lib = env
+    g = torch.Generator(device="cuda").manual_seed(M + N + K)
+    A = (torch.randn(M, K, device="cuda", generator=g) * 0.5).to(torch.bfloat16)
+    W = (torch.randn(N, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    assert torch.equal(_run(torch, lib, 0, A, W), _run(torch, lib, 2, A, W))
 
 
 def test_gemm_repeat_is_deterministic(env):
