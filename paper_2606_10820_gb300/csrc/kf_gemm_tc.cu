@@ -39,6 +39,7 @@ constexpr int kBK = 64;                 // one 128-byte swizzle atom of bf16
 
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kPersistWarps = 2 + kEpiWarps + 1;   // + a second TMA producer
 
 // per-row data of a tile, fetched by the epilogue warps during the mainloop
 struct EpiMeta {
@@ -70,16 +71,65 @@ __device__ __forceinline__ void epi_bar() {
 // ch: which of the quarter's two warps (alternate 64-column blocks, or
 // alternate halves of the rows when the tile has one block).
 template <int BN, int EPI>
+struct EpiRows {
+  static constexpr int NB = BN / 64;                  // 64-column blocks
+  static constexpr int NI = NB >= 2 ? 8 : 4;          // row groups per warp
+  static constexpr bool kAny = EPI == EPI_QKV || EPI == EPI_RESID;
+  // per row group of one block: QKV the RoPE cos / sin at the row's
+  // position, RESID the residual x (columns gc and gc + 32)
+  float4 a[kAny ? NI : 1], b[kAny ? NI : 1];
+};
+
+// the first 64-column block of this warp (NB >= 2: block ch, else block 0)
+template <int BN>
+__device__ __forceinline__ int epi_first_block(int ch) { return BN / 64 >= 2 ? ch : 0; }
+
+// Issue the global loads of the per-row data of block bb (all row groups at
+// once, so their latencies overlap); EPI_QKV reads meta->pos.
+template <int BN, int EPI>
+__device__ __forceinline__ void epi_rows_load(EpiRows<BN, EPI>& r, const TcArgs& g, const EpiMeta* meta, int m0,
+                                              int n0, int quarter, int ch, int lane, int bb) {
+  using R = EpiRows<BN, EPI>;
+  const int ibase = R::NB >= 2 ? 0 : ch * 4;
+  const int gr = lane >> 3, gc = (lane & 7) * 4;
+  const int c = bb * 64;
+  if (EPI == EPI_QKV) {
+    if (g.epi.cos_t && n0 + c < 2 * g.epi.dsec) {         // q and k rotate
+#pragma unroll
+      for (int ii = 0; ii < R::NI; ++ii) {
+        const int pos = meta->pos[quarter * 32 + gr + 4 * (ibase + ii)];
+        r.a[ii] = __ldg(reinterpret_cast<const float4*>(g.epi.cos_t + (size_t)pos * 32 + gc));
+        r.b[ii] = __ldg(reinterpret_cast<const float4*>(g.epi.sin_t + (size_t)pos * 32 + gc));
+      }
+    }
+  } else if (EPI == EPI_RESID) {
+#pragma unroll
+    for (int ii = 0; ii < R::NI; ++ii) {
+      const int row = m0 + quarter * 32 + gr + 4 * (ibase + ii);
+      const float* xp = g.epi.x + (size_t)row * g.epi.ldx + n0 + c + gc;
+      const bool okr = row < g.M && n0 + c + gc < g.N;
+      r.a[ii] = okr ? *reinterpret_cast<const float4*>(xp) : make_float4(0.f, 0.f, 0.f, 0.f);
+      r.b[ii] = (okr && n0 + c + 32 + gc < g.N) ? *reinterpret_cast<const float4*>(xp + 32)
+                                                : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+}
+
+// r holds the per-row data of the warp's first block on entry (epi_rows_load
+// with epi_first_block, issued before the accumulator wait)
+template <int BN, int EPI>
 __device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* meta, float* T, uint32_t lane_addr,
-                                             int m0, int n0, int quarter, int ch, int lane) {
-  constexpr int NB = BN / 64;                 // 64-column blocks
-  constexpr int NI = NB >= 2 ? 8 : 4;         // row groups per warp
-  const int b0 = NB >= 2 ? ch : 0;
+                                             int m0, int n0, int quarter, int ch, int lane, EpiRows<BN, EPI>& r) {
+  using R = EpiRows<BN, EPI>;
+  constexpr int NB = R::NB, NI = R::NI;
+  const int b0 = epi_first_block<BN>(ch);
   const int ibase = NB >= 2 ? 0 : ch * 4;
   const int gr = lane >> 3, gc = (lane & 7) * 4;
 #pragma unroll 1
   for (int bb = b0; bb < NB; bb += (NB >= 2 ? 2 : 1)) {
     const int c = bb * 64;
+    if (n0 + c >= g.N) break;                  // past the last column (warp-uniform)
+    if (bb != b0) epi_rows_load<BN, EPI>(r, g, meta, m0, n0, quarter, ch, lane, bb);
 #pragma unroll
     for (int h2 = 0; h2 < 2; ++h2) {
       float v[32];
@@ -89,20 +139,12 @@ __device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* met
         *reinterpret_cast<float4*>(T + lane * 68 + 32 * h2 + 4 * q) =
             make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
     }
-    // residuals of all this warp's rows first (EPI_RESID)
-    float4 xlo[EPI == EPI_RESID ? NI : 1], xhi[EPI == EPI_RESID ? NI : 1];
-    if (EPI == EPI_RESID) {
-#pragma unroll
-      for (int ii = 0; ii < NI; ++ii) {
-        const int row = m0 + quarter * 32 + gr + 4 * (ibase + ii);
-        const float* xp = g.epi.x + (size_t)row * g.epi.ldx + n0 + c + gc;
-        const bool okr = row < g.M && n0 + c + gc < g.N;
-        xlo[ii] = okr ? *reinterpret_cast<const float4*>(xp) : make_float4(0.f, 0.f, 0.f, 0.f);
-        xhi[ii] = (okr && n0 + c + 32 + gc < g.N) ? *reinterpret_cast<const float4*>(xp + 32)
-                                                  : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    }
     __syncwarp();
+    float4 bias_lo = make_float4(0.f, 0.f, 0.f, 0.f), bias_hi = bias_lo;
+    if (EPI == EPI_BIAS_GELU && g.epi.bias) {
+      bias_lo = __ldg(reinterpret_cast<const float4*>(g.epi.bias + n0 + c + gc));
+      if (n0 + c + 32 + gc < g.N) bias_hi = __ldg(reinterpret_cast<const float4*>(g.epi.bias + n0 + c + 32 + gc));
+    }
 #pragma unroll
     for (int ii = 0; ii < NI; ++ii) {
       const int rl = quarter * 32 + gr + 4 * (ibase + ii);   // row within the tile
@@ -111,18 +153,21 @@ __device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* met
       float4 lo = *reinterpret_cast<const float4*>(T + (rl - quarter * 32) * 68 + gc);
       float4 hi = *reinterpret_cast<const float4*>(T + (rl - quarter * 32) * 68 + 32 + gc);
       if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && ok && g.epi.ss_in) {
-        const float r = meta->rinv[rl];        // fused RMSNorm of the A rows
-        lo = scale4(lo, r);
-        hi = scale4(hi, r);
+        const float ri = meta->rinv[rl];        // fused RMSNorm of the A rows
+        lo = scale4(lo, ri);
+        hi = scale4(hi, ri);
       }
       float sq = 0.f;
       if (ok) {
         if (EPI == EPI_QKV) {
-          epi_qkv<__nv_bfloat16>(g.epi, row, meta->pos[rl], meta->aux[rl], n0 + c, gc, lo, hi);
+          epi_qkv_rot<__nv_bfloat16>(g.epi, row, meta->pos[rl], meta->aux[rl], n0 + c, gc, lo, hi, r.a[ii], r.b[ii]);
         } else if (EPI == EPI_RESID) {
-          if (n0 + c + gc < g.N) sq = epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + gc, lo, xlo[ii]);
+          if (n0 + c + gc < g.N) sq = epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + gc, lo, r.a[ii]);
           if (n0 + c + 32 + gc < g.N)
-            sq += epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + 32 + gc, hi, xhi[ii]);
+            sq += epi_resid4<__nv_bfloat16>(g.epi, row, n0 + c + 32 + gc, hi, r.b[ii]);
+        } else if (EPI == EPI_BIAS_GELU) {
+          sq = epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, add4(lo, bias_lo), g.N, false) +
+               epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, add4(hi, bias_hi), g.N, false);
         } else {
           sq = epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + gc, lo, g.N) +
                epi_vec4<__nv_bfloat16, EPI>(g.epi, row, n0 + c + 32 + gc, hi, g.N);
@@ -140,7 +185,8 @@ __device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* met
       }
     }
     __syncwarp();
-  }}
+  }
+}
 
 // ------------------------------------------------------------ the kernel
 // MT: 128-row M tiles per CTA, each with its own TMEM accumulator (2 only for
@@ -202,13 +248,22 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
+  // Producers: warp 0 and, for stages of several boxes, the last epilogue
+  // warps (idle until the accumulator is ready) each issue their share of a
+  // stage's TMA boxes.  One thread issues about one copy per 250 ns whatever
+  // its size, so copies from one thread cap the operand stream; warps issue
+  // side by side.  Box j of a stage: K atom j / (MT + 1); A box (M half
+  // j % (MT + 1)) or, for the last one, the W box.  Warp 0 arms each stage's
+  // barrier.  Weights are constant during a step: the first stages' W boxes
+  // stream in while the predecessor kernel finishes; the A boxes it produces
+  // are loaded after pdl_wait.
+  constexpr int NBOX = AT * (MT + 1);
+  constexpr int NPW = NBOX < 4 ? NBOX : 4;
+  const int pw = warp == 0 ? 0 : (warp > kThreads / 32 - NPW ? kThreads / 32 - warp : -1);
+  if (pw >= 0) {
     if (lane == 0) {
-      // Weights are constant during a step: the first stages' weight tiles
-      // stream in while the predecessor kernel finishes; the activation tiles
-      // it produces are loaded after pdl_wait.
       const int pre = min(nst, STAGES);
-      if (g.l2_next) {
+      if (pw == 0 && g.l2_next) {
         // this CTA's share of the next projection's weights, into L2 for the
         // kernel after this one (256-byte slices, one prefetch each of at
         // most 1 MiB)
@@ -220,38 +275,38 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
           prefetch_l2(g.l2_next + o, (uint32_t)(n & ~15ull));
         }
       }
+      // the boxes of stage i that this warp issues: W (w = true) or A boxes
+      auto issue = [&](int i, uint32_t sa, uint32_t full, bool w_boxes) {
+        const int na = min(AT, nkb - i * AT);
+        for (int j = pw; j < na * (MT + 1); j += NPW) {
+          const int a = j / (MT + 1), r = j % (MT + 1);
+          const int kc = (kb0 + i * AT + a) * kBK;
+          if (r == MT && w_boxes) tma_load_2d(sa + A_BYTES + a * B_ATOM, &map_w, full, kc, n0);
+          if (r < MT && !w_boxes) tma_load_2d(sa + (a * MT + r) * A_ATOM, &map_a, full, kc, m0 + r * kBM);
+        }
+      };
       for (int i = 0; i < pre; ++i) {
         const uint32_t full = smem_u32(&bars[i]);
-        const int na = min(AT, nkb - i * AT);
-        mbar_expect_tx(full, na * (MT * g.a_box + B_ATOM));
-        for (int a = 0; a < na; ++a)
-          tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_BYTES + a * B_ATOM, &map_w, full,
-                      (kb0 + i * AT + a) * kBK, n0);
+        if (pw == 0) mbar_expect_tx(full, min(AT, nkb - i * AT) * (MT * g.a_box + B_ATOM));
+        issue(i, smem_u32(smem + i * STAGE_BYTES), full, true);
       }
       pdl_wait();
-      for (int i = 0; i < pre; ++i) {
-        const int na = min(AT, nkb - i * AT);
-        for (int a = 0; a < na; ++a)
-          for (int mh = 0; mh < MT; ++mh)
-            tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + (a * MT + mh) * A_ATOM, &map_a,
-                        smem_u32(&bars[i]), (kb0 + i * AT + a) * kBK, m0 + mh * kBM);
-      }
+      for (int i = 0; i < pre; ++i) issue(i, smem_u32(smem + i * STAGE_BYTES), smem_u32(&bars[i]), false);
       for (int i = pre; i < nst; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (i / STAGES) & 1;
         if (!mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, g.d_err)) break;
         const uint32_t full = smem_u32(&bars[s]);
-        const int na = min(AT, nkb - i * AT);
-        mbar_expect_tx(full, na * (MT * g.a_box + B_ATOM));
+        if (pw == 0) mbar_expect_tx(full, min(AT, nkb - i * AT) * (MT * g.a_box + B_ATOM));
         const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
-        for (int a = 0; a < na; ++a) {
-          const int kc = (kb0 + i * AT + a) * kBK;
-          for (int mh = 0; mh < MT; ++mh)
-            tma_load_2d(sa + (a * MT + mh) * A_ATOM, &map_a, full, kc, m0 + mh * kBM);
-          tma_load_2d(sa + A_BYTES + a * B_ATOM, &map_w, full, kc, n0);
-        }
+        issue(i, sa, full, true);
+        issue(i, sa, full, false);
       }
     }
+    __syncwarp();
+  }
+  if (warp == 0) {
+    // producer only
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, BN);
@@ -307,14 +362,20 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         meta->aux[et] = page;
       }
     }
+    const int rbase = m0 + quarter * 32;
+    const bool active = rbase < g.M;          // warp-uniform
+    // the per-row data of the warp's first block, before the accumulator is
+    // ready (QKV: after the positions above are published)
+    EpiRows<BN, EPI> rows;
+    const bool vec = EPI != EPI_HEAD && g.splits == 1 && active;
+    if (EPI == EPI_QKV) epi_bar();
+    if (vec) epi_rows_load<BN, EPI>(rows, g, meta, m0, n0, quarter, ch, lane, epi_first_block<BN>(ch));
     // one waiter, result broadcast: every epilogue thread takes the same path
     if (et == 0) s_flag[1] = mbar_wait(smem_u32(&bars[2 * STAGES]), 0, g.d_err) ? 1 : 0;
     epi_bar();
     const bool ready = s_flag[1] != 0;
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
-    const int rbase = m0 + quarter * 32;
-    const bool active = rbase < g.M;          // warp-uniform
     if (ready && active) {
       if (g.splits > 1) {
         // this split's partial: rows of the tile in the CTA's own shared
@@ -346,7 +407,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
       } else {
         // per epilogue warp a 32 x 68 fp32 block in the idle pipeline stages
         epi_vec_tile<BN, EPI>(g, meta, reinterpret_cast<float*>(smem) + (warp - 2) * (32 * 68), lane_addr, m0, n0,
-                              quarter, ch, lane);
+                              quarter, ch, lane, rows);
       }
     }
   }
@@ -371,7 +432,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
         const int pr = idx % GQ;
         const int blk = (pr / 8) * 64, g4 = (pr % 8) * 4;
         const int row = m0 + rr;
-        if (row >= g.M) continue;
+        if (row >= g.M || n0 + blk >= g.N) continue;
         float4 lo = make_float4(0.f, 0.f, 0.f, 0.f), hi = lo;
         const uint32_t off = (uint32_t)((rr * (BN + 4) + blk + g4) * 4);
         for (int sp = 0; sp < S; ++sp) {
@@ -475,7 +536,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
 // cost about one mainloop each instead of a mainloop plus an epilogue.  The
 // epilogue stages through its own shared memory (the ring stays busy).
 template <int BN, int STAGES, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kPersistWarps * 32, 1)
 k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_w,
                   TcArgs g) {
   constexpr uint32_t A_ATOM = kBM * kBK * 2;
@@ -526,50 +587,69 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
+  if (warp == 0 || warp == kPersistWarps - 1) {
+    // two producers issue side by side (one thread issues about one TMA copy
+    // per 250 ns): warp 0 arms each stage's barrier and loads its A box, the
+    // last warp loads its W box.  The first tile's W boxes stream in while the
+    // predecessor kernel finishes.
     if (lane == 0) {
+      const bool wp = warp != 0;
       uint32_t stage = 0;
       bool first = true;
       for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
         const int m0 = (t / n_tiles) * kBM, n0 = (t % n_tiles) * BN;
         int i0 = 0;
         if (first) {
-          // the first stages' weights before the predecessor kernel is done
           const int pre = min(nkb, STAGES);
           for (int i = 0; i < pre; ++i) {
-            mbar_expect_tx(smem_u32(&full[i]), g.a_box + B_ATOM);
-            tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_ATOM, &map_w, smem_u32(&full[i]), i * kBK, n0);
+            if (!wp) mbar_expect_tx(smem_u32(&full[i]), g.a_box + B_ATOM);
+            else tma_load_2d(smem_u32(smem + i * STAGE_BYTES) + A_ATOM, &map_w, smem_u32(&full[i]), i * kBK, n0);
           }
-          pdl_wait();
-          for (int i = 0; i < pre; ++i)
-            tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &map_a, smem_u32(&full[i]), i * kBK, m0);
+          if (!wp) {
+            pdl_wait();
+            for (int i = 0; i < pre; ++i)
+              tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &map_a, smem_u32(&full[i]), i * kBK, m0);
+          }
           i0 = pre;
           first = false;
         }
+        bool live = true;
         for (int i = i0; i < nkb; ++i) {
           const uint32_t sc = stage + i, s = sc % STAGES;
-          if (!mbar_wait(smem_u32(&empty[s]), ((sc / STAGES) & 1) ^ 1, g.d_err)) break;
+          if (!mbar_wait(smem_u32(&empty[s]), ((sc / STAGES) & 1) ^ 1, g.d_err)) {
+            live = false;
+            break;
+          }
           const uint32_t fb = smem_u32(&full[s]);
-          mbar_expect_tx(fb, g.a_box + B_ATOM);
           const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
-          tma_load_2d(sa, &map_a, fb, i * kBK, m0);
-          tma_load_2d(sa + A_ATOM, &map_w, fb, i * kBK, n0);
+          if (!wp) {
+            mbar_expect_tx(fb, g.a_box + B_ATOM);
+            tma_load_2d(sa, &map_a, fb, i * kBK, m0);
+          } else {
+            tma_load_2d(sa + A_ATOM, &map_w, fb, i * kBK, n0);
+          }
         }
+        if (!live) break;
         stage += nkb;
       }
     }
+    __syncwarp();
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kBM, BN);
       uint32_t stage = 0, ti = 0;
-      for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++ti) {
+      bool ok = true;   // a timed-out wait ends this CTA's tiles
+      for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++ti) {
         const uint32_t buf = ti & 1;
-        mbar_wait(smem_u32(&acce[buf]), ((ti >> 1) & 1) ^ 1, g.d_err);
+        if (!mbar_wait(smem_u32(&acce[buf]), ((ti >> 1) & 1) ^ 1, g.d_err)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t d = tmem + buf * BN;
         for (int i = 0; i < nkb; ++i, ++stage) {
           const uint32_t s = stage % STAGES;
-          mbar_wait(smem_u32(&full[s]), (stage / STAGES) & 1, g.d_err);
+          if (!mbar_wait(smem_u32(&full[s]), (stage / STAGES) & 1, g.d_err)) {
+            ok = false;
+            break;
+          }
           asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
           const uint32_t sa = smem_u32(smem + s * STAGE_BYTES);
 #pragma unroll
@@ -577,7 +657,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
             mma_bf16(d, sdesc(sa + kk * 32), sdesc(sa + A_ATOM + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
           mma_commit(smem_u32(&empty[s]));
         }
-        mma_commit(smem_u32(&accf[buf]));
+        if (ok) mma_commit(smem_u32(&accf[buf]));
       }
     }
   } else {
@@ -585,7 +665,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
     const int ch = (warp - 2) >> 2;
     const int et = threadIdx.x - 64;
     pdl_wait();
-    uint32_t ti = 0;
+    uint32_t ti = 0;   // epilogue warps 2 .. kEpiWarps + 1
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++ti) {
       const uint32_t buf = ti & 1;
       const int m0 = (t / n_tiles) * kBM, n0 = (t % n_tiles) * BN;
@@ -611,12 +691,18 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
           meta->aux[et] = page;
         }
       }
+      // the first block's per-row data before the accumulator is ready
+      const bool active = m0 + quarter * 32 < g.M;   // warp-uniform
+      EpiRows<BN, EPI> rows;
+      if (EPI == EPI_QKV) epi_bar();
+      if (active) epi_rows_load<BN, EPI>(rows, g, meta, m0, n0, quarter, ch, lane, epi_first_block<BN>(ch));
       if (et == 0) s_flag[0] = mbar_wait(smem_u32(&accf[buf]), (ti >> 1) & 1, g.d_err) ? 1 : 0;
       epi_bar();
+      if (!s_flag[0]) break;   // timed out: the MMA warp has stopped too
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t lane_addr = tmem + buf * BN + ((uint32_t)(quarter * 32) << 16);
-      if (s_flag[0] && m0 + quarter * 32 < g.M)
-        epi_vec_tile<BN, EPI>(g, meta, stg + (warp - 2) * (32 * 68), lane_addr, m0, n0, quarter, ch, lane);
+      if (active)
+        epi_vec_tile<BN, EPI>(g, meta, stg + (warp - 2) * (32 * 68), lane_addr, m0, n0, quarter, ch, lane, rows);
       // every warp has read the accumulator: the MMA warp may refill it
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       epi_bar();
@@ -782,7 +868,7 @@ static int launch_persist_epi(const GemmDesc& g, int* d_err, int num_sms, cudaSt
   a.d_err = d_err; a.epi = g.epi;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(std::min(tiles, num_sms));
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kPersistWarps * 32);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute at[1];
@@ -850,6 +936,10 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
   // tile keeps a fourth pipeline stage and has nothing to overlap.  The
   // LM-head records keep their kernel, which streams each weight tile once
   // per 256 rows.
+  // (One wave of 256-wide tiles stays one CTA per tile even where it leaves
+  // SMs idle: persistent 128-wide tiles for the OWT-shaped O projection and
+  // MLP-down at 4096 rows, 192 tiles on 152 SMs, were 1.3-1.6x slower; each
+  // SM streams twice the A bytes per flop, and the stream is the limit.)
   if (g.epi.kind != EPI_HEAD && !(g_gemm_flags & kGemmNoPersist) && ceil_div(g.N, 256) * m_tiles > num_sms)
     return launch_persist<256, 3>(g, d_err, num_sms, s);
   return launch_bn<256, 4, 1>(g, d_err, num_sms, s);

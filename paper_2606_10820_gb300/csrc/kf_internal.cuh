@@ -174,17 +174,17 @@ __device__ __forceinline__ float row_rinv(const Epi& e, int row) {
 
 // EPI_QKV for one row at position pos whose KV page is `page` (-1: invalid,
 // already flagged): lo = columns col0+gc .. +3 and hi = the same columns + 32
-// of one 64-wide head block (col0 % 64 == 0, head_dim 64).  Rotates the
-// pairs (i, i + 32) of q and k at the row's position and stores q, k, v.
+// of one 64-wide head block (col0 % 64 == 0, col0 < 3 * dsec, head_dim 64).
+// Rotates the pairs (i, i + 32) of q and k at the row's position, with
+// c4 / s4 = cos / sin of the angles gc .. gc + 3 at pos (read by the caller:
+// cos_t / sin_t [pos][gc]), and stores q, k, v.
 template <typename TA>
-__device__ __forceinline__ void epi_qkv(const Epi& e, int row, int pos, int page, int col0, int gc,
-                                        float4 lo, float4 hi) {
+__device__ __forceinline__ void epi_qkv_rot(const Epi& e, int row, int pos, int page, int col0, int gc,
+                                            float4 lo, float4 hi, float4 c4, float4 s4) {
   const int sec = col0 / e.dsec;                 // 0 q, 1 k, 2 v
   const int h = (col0 - sec * e.dsec) >> 6;
   float a[4] = {lo.x, lo.y, lo.z, lo.w}, b[4] = {hi.x, hi.y, hi.z, hi.w};
   if (sec < 2 && e.cos_t) {
-    const float4 c4 = __ldg(reinterpret_cast<const float4*>(e.cos_t + (size_t)pos * 32 + gc));
-    const float4 s4 = __ldg(reinterpret_cast<const float4*>(e.sin_t + (size_t)pos * 32 + gc));
     const float c[4] = {c4.x, c4.y, c4.z, c4.w}, sn[4] = {s4.x, s4.y, s4.z, s4.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -205,6 +205,18 @@ __device__ __forceinline__ void epi_qkv(const Epi& e, int row, int pos, int page
             (size_t)(pos % kPage) * 64 + gc;
   st_ta4(dst, make_float4(a[0], a[1], a[2], a[3]));
   st_ta4(dst + 32, make_float4(b[0], b[1], b[2], b[3]));
+}
+
+// the same, reading the angles' cos / sin itself
+template <typename TA>
+__device__ __forceinline__ void epi_qkv(const Epi& e, int row, int pos, int page, int col0, int gc,
+                                        float4 lo, float4 hi) {
+  float4 c4 = make_float4(1.f, 1.f, 1.f, 1.f), s4 = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (e.cos_t && col0 < 2 * e.dsec) {
+    c4 = __ldg(reinterpret_cast<const float4*>(e.cos_t + (size_t)pos * 32 + gc));
+    s4 = __ldg(reinterpret_cast<const float4*>(e.sin_t + (size_t)pos * 32 + gc));
+  }
+  epi_qkv_rot<TA>(e, row, pos, page, col0, gc, lo, hi, c4, s4);
 }
 
 template <typename TA>
@@ -314,14 +326,15 @@ __device__ __forceinline__ float epi_resid4(const Epi& e, int row, int col, floa
 }
 
 template <typename TA, int EPI>
-__device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4 v, int N) {
+__device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4 v, int N,
+                                         bool add_bias = true) {
   if (col >= N) return 0.f;
   if (EPI == EPI_STORE) {
     st_ta4(reinterpret_cast<TA*>(e.out) + (size_t)row * e.ldo + col, v);
   } else if (EPI == EPI_STORE_F32) {
     *reinterpret_cast<float4*>(e.outf + (size_t)row * e.ldo + col) = v;
   } else if (EPI == EPI_BIAS_GELU) {
-    if (e.bias) {
+    if (e.bias && add_bias) {   // (false: the caller has added it)
       float4 b = __ldg(reinterpret_cast<const float4*>(e.bias + col));
       v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
     }
@@ -362,6 +375,9 @@ __device__ __forceinline__ float epi_vec4(const Epi& e, int row, int col, float4
 
 __device__ __forceinline__ float4 scale4(float4 v, float r) {
   return make_float4(v.x * r, v.y * r, v.z * r, v.w * r);
+}
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
 // ---------------------------------------------------------------- launches
