@@ -59,6 +59,7 @@ struct kf_ctx {
   float* rope_cos = nullptr;
   float* rope_sin = nullptr;
   double* noise_freq = nullptr;
+  float* tau_feat = nullptr;   // [d]: cos | sin of noise_scale * tau * noise_freq
   // paged KV
   void* kv = nullptr;
   int n_pages = 0, max_pages = 0;
@@ -72,6 +73,13 @@ struct kf_ctx {
   int B = 0, P = 0, last_nh = 0;
   std::vector<int> h_len, h_len0;
   int32_t *d_len = nullptr, *d_len0 = nullptr, *d_pending = nullptr, *d_pending0 = nullptr;
+  // decode attention visits the sequences longest first (d_order: a
+  // permutation of 0..B-1 by decreasing cached length, ties by index); every
+  // step adds the same count to every length, so only prefill, admit and
+  // rewind change it
+  int32_t* d_order = nullptr;
+  std::vector<int32_t> h_order;
+  bool order_dirty = true;
   int pend_stride = 8;
   // workspaces
   int R_cap = 0, NR_cap = 0, prefill_rows = 0;
@@ -300,6 +308,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
     a.uniform_rows = uniform_rows; a.out = c->attn; a.part_o = c->part_o; a.part_ml = c->part_ml;
     a.R = R; a.n_split = n_split; a.keys_per_split = kps; a.d_err = c->d_err;
     a.len = groups ? nullptr : c->d_len;   // decode: keys below it are stable during the step
+    a.order = groups || !mma_attn ? nullptr : c->d_order;   // longest sequences first
     a.split_count = c->split_count;
     prof_begin(c, KF_KIND_ATTENTION);
     bool merged = false;
@@ -352,7 +361,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
                        c->row_pos, c->V, d, c->x, c->fused ? c->xn : nullptr,
                        c->fused ? c->ss : nullptr, c->d_err, s);
   if (k > 0)
-    launch_noise_feat(c->bf16, B * k, noise, c->noise_freq, c->cfg.tau, c->cfg.noise_scale, d,
+    launch_noise_feat(c->bf16, B * k, noise, c->noise_freq, c->tau_feat, c->cfg.noise_scale, d,
                       c->nfeat, s);
   prof_end(c);
   if (k > 0) {
@@ -589,10 +598,17 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
     if ((r = fbuf(&c->rope_cos, cs.size())) || (r = fbuf(&c->rope_sin, sn.size()))) return bail(r);
     std::vector<double> fr(d / 2);
     for (int t = 0; t < d / 2; ++t) fr[t] = std::exp(-std::log(1e4) * t / (d / 2));
-    if ((r = dalloc(c, &c->noise_freq, fr.size() * 8))) return bail(r);
+    std::vector<float> tf(d);
+    for (int t = 0; t < d / 2; ++t) {
+      const double ang = (double)cfg.noise_scale * (double)cfg.tau * fr[t];
+      tf[t] = (float)std::cos(ang);
+      tf[d / 2 + t] = (float)std::sin(ang);
+    }
+    if ((r = dalloc(c, &c->noise_freq, fr.size() * 8)) || (r = fbuf(&c->tau_feat, tf.size()))) return bail(r);
     if (cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(c->noise_freq, fr.data(), fr.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaMemcpy(c->noise_freq, fr.data(), fr.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(c->tau_feat, tf.data(), tf.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
       cuda_fail(c, cudaGetLastError(), "table upload");
       return bail(KF_E_CUDA);
     }
@@ -617,6 +633,7 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
   c->R_cap = std::max(round_up(MB * 2 * MK, 128), c->prefill_rows);
   const int R = c->R_cap;
   if ((r = dalloc(c, &c->d_len, MB * 4)) || (r = dalloc(c, &c->d_len0, MB * 4)) ||
+      (r = dalloc(c, &c->d_order, MB * 4)) ||
       (r = dalloc(c, &c->d_pending, (size_t)MB * MK * 4)) ||
       (r = dalloc(c, &c->d_pending0, (size_t)MB * MK * 4)) ||
       (r = dalloc(c, &c->x, (size_t)R * d * 4)) || (r = wbuf(&c->xn, (size_t)R * d)) ||
@@ -755,6 +772,7 @@ int kf_prefill(kf_ctx* c, int32_t B, const int32_t* tokens, const int32_t* lens)
     off += ln[b];
   }
   c->h_len0 = c->h_len;
+  c->order_dirty = true;
   std::vector<int32_t> hl(c->h_len.begin(), c->h_len.end());
   KF_CUDA(cudaMemcpyAsync(c->d_len, hl.data(), B * 4, cudaMemcpyHostToDevice, c->stream));
   KF_CUDA(cudaMemcpyAsync(c->d_len0, hl.data(), B * 4, cudaMemcpyHostToDevice, c->stream));
@@ -828,6 +846,7 @@ int kf_admit(kf_ctx* c, int32_t n, const int32_t* slots, const int32_t* tokens, 
                             (size_t)P * 4, cudaMemcpyHostToDevice, c->stream));
     KF_CUDA(cudaMemcpyAsync(c->d_len + sl[i], nl.data() + i, 4, cudaMemcpyHostToDevice, c->stream));
     c->h_len[sl[i]] = nl[i];
+    c->order_dirty = true;
   }
   KF_CUDA(cudaStreamSynchronize(c->stream));
   int err = 0;
@@ -835,6 +854,21 @@ int kf_admit(kf_ctx* c, int32_t n, const int32_t* slots, const int32_t* tokens, 
   if (err) return fail(c, KF_E_DEVICE, "device error flag " + std::to_string(err) + " in admit");
   c->admitted = true;
   c->have_step = false;
+  return KF_OK;
+}
+
+// the attention's sequence order for the current lengths (uploaded when
+// prefill, admit or rewind changed them)
+static int sync_order(kf_ctx* c) {
+  if (!c->order_dirty) return KF_OK;
+  const int B = c->B;
+  c->h_order.resize(B);
+  for (int b = 0; b < B; ++b) c->h_order[b] = b;
+  std::stable_sort(c->h_order.begin(), c->h_order.end(),
+                   [&](int32_t x, int32_t y) { return c->h_len[x] > c->h_len[y]; });
+  KF_CUDA(cudaMemcpyAsync(c->d_order, c->h_order.data(), (size_t)B * 4, cudaMemcpyHostToDevice, c->stream));
+  // the copy reads pageable memory: it has been staged when it returns
+  c->order_dirty = false;
   return KF_OK;
 }
 
@@ -852,6 +886,7 @@ int kf_teacher_step(kf_ctx* c, int32_t B, int32_t k, const float* noise, int32_t
     KF_TRY(ensure_pages(c, b, c->h_len[b] + P + k - 1, &dirty));
     if (dirty) KF_TRY(upload_page_row(c, b));
   }
+  KF_TRY(sync_order(c));
   // noise [B][k] -> [k][B]: sub-step j reads a contiguous column
   for (int j = 0; j < k; ++j)
     KF_CUDA(cudaMemcpy2DAsync(c->noise + (size_t)j * B, 4, noise + j, (size_t)k * 4, 4, B, cudaMemcpyDefault,
@@ -920,6 +955,7 @@ static int step_common(kf_ctx* c, int32_t B, int32_t k, const float* noise, int3
     KF_TRY(ensure_pages(c, b, c->h_len[b] + P + k - 1, &dirty));
     if (dirty) KF_TRY(upload_page_row(c, b));
   }
+  KF_TRY(sync_order(c));
   KF_CUDA(cudaMemcpyAsync(c->noise, noise, (size_t)B * nout * 4, cudaMemcpyDefault, c->stream));
   bool use_graph = !profile && !(c->cfg.flags & KF_FLAG_NO_GRAPH);
   if (use_graph) {
@@ -1057,6 +1093,7 @@ int kf_rewind(kf_ctx* c) {
   KF_CUDA(cudaMemcpyAsync(c->d_pending, c->d_pending0, (size_t)c->B * c->pend_stride * 4,
                           cudaMemcpyDeviceToDevice, c->stream));
   c->h_len = c->h_len0;
+  c->order_dirty = true;
   c->P = 1;
   c->have_step = false;
   return KF_OK;

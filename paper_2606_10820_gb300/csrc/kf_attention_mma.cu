@@ -128,7 +128,8 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
   const bool early = a.len != nullptr && a.groups == nullptr;
   int b, row0, nr, n_keys, stable;
   if (early) {
-    b = gi; row0 = gi * a.uniform_rows; nr = a.uniform_rows;
+    b = a.order ? __ldg(a.order + gi) : gi;
+    row0 = b * a.uniform_rows; nr = a.uniform_rows;
     stable = a.len[b];                       // committed length: positions row_pos of the step
     n_keys = stable + nr;
   } else {
@@ -137,7 +138,8 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
       const int4 gg = a.groups[gi];
       b = gg.x; row0 = gg.y; nr = gg.z;
     } else {
-      b = gi; row0 = gi * a.uniform_rows; nr = a.uniform_rows;
+      b = a.order ? __ldg(a.order + gi) : gi;
+      row0 = b * a.uniform_rows; nr = a.uniform_rows;
     }
     n_keys = a.row_pos[row0 + nr - 1] + 1;
     stable = 0;
@@ -171,6 +173,14 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // zeros before the copies
   __syncthreads();
 
+  // One buffer: lane i of warp 0 holds the page id of page i of the tile at
+  // pf_kt, read one tile ahead so that its latency overlaps the compute of
+  // the tile before (the page table does not change during the step)
+  int pf_page = -1, pf_kt = -1;
+  auto page_id = [&](int kq) -> int {
+    const int pi = kq / kPage;
+    return kq < k_end && pi < a.max_pages ? __ldg(a.page_table + (size_t)b * a.max_pages + pi) : -1;
+  };
   // Copies of the pages of the tile at kt whose first key lies in
   // [key_lo, key_hi) (multiples of the page size) into buffer buf, by lanes
   // 0..7 of warp 0 (one page each).  The bytes are added to the buffer's
@@ -180,10 +190,16 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
     const int kq = kt + lane * kPage;         // first key of this lane's page
     int page = -1;
     bool go = false;
+    if constexpr (NBUF == 1) {
+      if (lane < kTile / kPage && pf_kt != kt) {
+        pf_page = page_id(kq);
+        pf_kt = kt;
+      }
+    }
     if (lane < kTile / kPage && kq < k_end && kq >= key_lo && kq < key_hi) {
       const int pi = kq / kPage;
       if constexpr (NBUF == 1)
-        page = pi < a.max_pages ? __ldg(a.page_table + (size_t)b * a.max_pages + pi) : -1;
+        page = pf_page;
       else
         page = pi - pg0 < n_pg ? s_pg[pi - pg0] : -1;
       go = page >= 0 && page < a.n_pages;
@@ -204,6 +220,13 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
       const uint32_t off = (uint32_t)(buf * kTileBytes + lane * kPageBytes);
       tma_load_2d(smem_u32(Ks) + off, &map_kv, bar, 0, row);
       tma_load_2d(smem_u32(Vs) + off, &map_kv, bar, 0, row + a.H * kPage);
+    }
+    if constexpr (NBUF == 1) {
+      // the next tile's page ids, consumed at its issue after this tile's compute
+      if (arrive && lane < kTile / kPage && kt + kTile < k_end) {
+        pf_page = page_id(kt + kTile + lane * kPage);
+        pf_kt = kt + kTile;
+      }
     }
   };
 

@@ -41,6 +41,9 @@ constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kPersistWarps = 2 + kEpiWarps + 1;   // + a second TMA producer
 
+// TMEM columns to allocate for n accumulator columns: a power of two >= 32
+__host__ __device__ constexpr int tmem_alloc_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 128 : n <= 256 ? 256 : 512; }
+
 // per-row data of a tile, fetched by the epilogue warps during the mainloop
 struct EpiMeta {
   float rinv[kBM];   // fused RMSNorm scale of the A row
@@ -61,6 +64,32 @@ struct TcArgs {
 
 __device__ __forceinline__ void epi_bar() {
   asm volatile("bar.sync 1, %0;" ::"n"(32 * kEpiWarps) : "memory");
+}
+
+// the per-row data of tile row et (row m0 + et): RMSNorm scale of the A row
+// (EPI_QKV, EPI_BIAS_GELU with ss_in), position and KV page (EPI_QKV; an
+// out-of-range page is flagged and stored as -1)
+template <int EPI>
+__device__ __forceinline__ void fill_meta(EpiMeta* meta, const TcArgs& g, int m0, int et) {
+  const int row = m0 + et;
+  const bool in = row < g.M;
+  if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in) meta->rinv[et] = in ? row_rinv(g.epi, row) : 0.f;
+  if (EPI == EPI_QKV) {
+    int pos = 0, page = -1;
+    if (in) {
+      pos = __ldg(g.epi.row_pos + row);
+      const int pi = pos / kPage;
+      page = pi < g.epi.max_pages
+                 ? __ldg(g.epi.page_table + (size_t)__ldg(g.epi.row_seq + row) * g.epi.max_pages + pi)
+                 : -1;
+      if (page < 0 || page >= g.epi.n_pages) {
+        page = -1;
+        atomicOr(g.epi.d_err, kErrBadPage);
+      }
+    }
+    meta->pos[et] = pos;
+    meta->aux[et] = page;
+  }
 }
 
 // The vector epilogue of one 128 x BN accumulator tile (one warp's share):
@@ -118,7 +147,8 @@ __device__ __forceinline__ void epi_rows_load(EpiRows<BN, EPI>& r, const TcArgs&
 // r holds the per-row data of the warp's first block on entry (epi_rows_load
 // with epi_first_block, issued before the accumulator wait)
 template <int BN, int EPI>
-__device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* meta, float* T, uint32_t lane_addr,
+__device__ __forceinline__ void epi_vec_tile(const TcArgs& g, const EpiMeta* meta, float* __restrict__ T,
+                                             uint32_t lane_addr,
                                              int m0, int n0, int quarter, int ch, int lane, EpiRows<BN, EPI>& r) {
   using R = EpiRows<BN, EPI>;
   constexpr int NB = R::NB, NI = R::NI;
@@ -201,7 +231,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   constexpr uint32_t B_ATOM = BN * kBK * 2;             // one BN x 64 W box
   constexpr uint32_t A_BYTES = AT * MT * A_ATOM;        // [atom][M tile] A boxes
   constexpr uint32_t STAGE_BYTES = AT * (MT * A_ATOM + B_ATOM);   // [A boxes][W atoms]
-  constexpr int TMEM_COLS = MT * BN;
+  constexpr int TMEM_COLS = tmem_alloc_cols(MT * BN);
+  static_assert(MT * BN <= 512 && BN % 16 == 0 && BN <= 256, "a 128 x BN MMA and its accumulators");
   static_assert(MT == 1 || EPI == EPI_HEAD, "two M tiles per CTA only for the LM-head records");
   static_assert(kEpiWarps * 32 * 68 * 4 <= STAGES * STAGE_BYTES &&
                     kBM * (BN + 4) * 4 <= STAGES * STAGE_BYTES,
@@ -340,28 +371,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
     const int et = threadIdx.x - 64;              // 0 .. 32*kEpiWarps-1
     pdl_wait();
     // the tile's per-row data, while the mainloop runs
-    if (et < kBM) {
-      const int row = m0 + et;
-      const bool in = row < g.M;
-      if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in)
-        meta->rinv[et] = in ? row_rinv(g.epi, row) : 0.f;
-      if (EPI == EPI_QKV) {
-        int pos = 0, page = -1;
-        if (in) {
-          pos = __ldg(g.epi.row_pos + row);
-          const int pi = pos / kPage;
-          page = pi < g.epi.max_pages
-                     ? __ldg(g.epi.page_table + (size_t)__ldg(g.epi.row_seq + row) * g.epi.max_pages + pi)
-                     : -1;
-          if (page < 0 || page >= g.epi.n_pages) {
-            page = -1;
-            atomicOr(g.epi.d_err, kErrBadPage);
-          }
-        }
-        meta->pos[et] = pos;
-        meta->aux[et] = page;
-      }
-    }
+    if (et < kBM) fill_meta<EPI>(meta, g, m0, et);
     const int rbase = m0 + quarter * 32;
     const bool active = rbase < g.M;          // warp-uniform
     // the per-row data of the warp's first block, before the accumulator is
@@ -543,7 +553,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
   constexpr uint32_t B_ATOM = BN * kBK * 2;
   constexpr uint32_t STAGE_BYTES = A_ATOM + B_ATOM;
   constexpr uint32_t STG_BYTES = kEpiWarps * 32 * 68 * 4;
-  constexpr int TMEM_COLS = 2 * BN;
+  constexpr int TMEM_COLS = tmem_alloc_cols(2 * BN);
   static_assert(EPI != EPI_HEAD, "the LM-head records keep their two-M-tile kernel");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -670,27 +680,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
       const uint32_t buf = ti & 1;
       const int m0 = (t / n_tiles) * kBM, n0 = (t % n_tiles) * BN;
       // the tile's per-row data while its mainloop runs
-      if (et < kBM) {
-        const int row = m0 + et;
-        const bool in = row < g.M;
-        if ((EPI == EPI_QKV || EPI == EPI_BIAS_GELU) && g.epi.ss_in) meta->rinv[et] = in ? row_rinv(g.epi, row) : 0.f;
-        if (EPI == EPI_QKV) {
-          int pos = 0, page = -1;
-          if (in) {
-            pos = __ldg(g.epi.row_pos + row);
-            const int pi = pos / kPage;
-            page = pi < g.epi.max_pages
-                       ? __ldg(g.epi.page_table + (size_t)__ldg(g.epi.row_seq + row) * g.epi.max_pages + pi)
-                       : -1;
-            if (page < 0 || page >= g.epi.n_pages) {
-              page = -1;
-              atomicOr(g.epi.d_err, kErrBadPage);
-            }
-          }
-          meta->pos[et] = pos;
-          meta->aux[et] = page;
-        }
-      }
+      if (et < kBM) fill_meta<EPI>(meta, g, m0, et);
       // the first block's per-row data before the accumulator is ready
       const bool active = m0 + quarter * 32 < g.M;   // warp-uniform
       EpiRows<BN, EPI> rows;
@@ -936,10 +926,15 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
   // tile keeps a fourth pipeline stage and has nothing to overlap.  The
   // LM-head records keep their kernel, which streams each weight tile once
   // per 256 rows.
-  // (One wave of 256-wide tiles stays one CTA per tile even where it leaves
-  // SMs idle: persistent 128-wide tiles for the OWT-shaped O projection and
-  // MLP-down at 4096 rows, 192 tiles on 152 SMs, were 1.3-1.6x slower; each
-  // SM streams twice the A bytes per flop, and the stream is the limit.)
+  // One wave of 256-wide tiles that leaves SMs idle, where 192-wide tiles
+  // still fit one wave: the narrower tiles (the OWT-shaped O projection and
+  // MLP-down at 4096 rows: 128 CTAs of 128 x 192 instead of 96 of 128 x 256;
+  // each streams 17 % fewer bytes per CTA).  (Persistent 128-wide tiles for
+  // those two, 192 tiles on 152 SMs, were 1.3-1.6x slower: a 128 x 128 tile
+  // streams twice the A bytes per flop, and the stream is the limit.)
+  if (ceil_div(g.N, 256) * m_tiles <= num_sms && ceil_div(g.N, 192) * m_tiles <= num_sms &&
+      ceil_div(g.N, 192) > ceil_div(g.N, 256))
+    return launch_bn<192, 5, 1>(g, d_err, num_sms, s);
   if (g.epi.kind != EPI_HEAD && !(g_gemm_flags & kGemmNoPersist) && ceil_div(g.N, 256) * m_tiles > num_sms)
     return launch_persist<256, 3>(g, d_err, num_sms, s);
   return launch_bn<256, 4, 1>(g, d_err, num_sms, s);

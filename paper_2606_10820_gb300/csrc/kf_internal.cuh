@@ -457,6 +457,10 @@ struct AttnArgs {
   int pg_cap = 0;                // pages of one CTA's key range (set by the launcher)
   int* split_count = nullptr;    // [groups][H] zeroed counters: the warp-MMA kernel merges
                                  // its own splits (no k_attn_combine launch)
+  const int32_t* order = nullptr;  // uniform groups: group g is sequence order[g] (a
+                                   // permutation, longest first: each head's longest CTAs
+                                   // start first and the grid's last wave holds the
+                                   // shortest), or NULL
 };
 // max_keys: the most keys any row of the launch can see (max_len bound)
 void launch_attention(bool bf16, const AttnArgs& a, int n_groups, int max_keys, cudaStream_t s);
@@ -483,7 +487,7 @@ void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* t
                          void* xb, float* ss, int* d_err, cudaStream_t s);
 void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, size_t total,
                        cudaStream_t s);
-void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
+void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, const float* tau_feat,
                        float scale, int d, void* feat, cudaStream_t s);
 void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
                     const float* g, float eps, void* out, cudaStream_t s);

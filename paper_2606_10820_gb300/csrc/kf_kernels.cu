@@ -155,33 +155,33 @@ __device__ __forceinline__ void sincos_reduced(double ang, float* s, float* c) {
   sincosf(r, s, c);
 }
 
+// tau_feat: the temperature's encoding [cos | sin] of scale * tau * freq, the
+// same for every row (computed once per context)
 template <typename TA>
 __global__ void k_noise_feat(int n, const float* __restrict__ noise, const double* __restrict__ freq,
-                             float tau, float scale, int d, TA* __restrict__ feat) {
+                             const float* __restrict__ tau_feat, float scale, int d, TA* __restrict__ feat) {
   pdl_trigger();
   pdl_wait();
   int half = d / 2;
   int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= n * half) return;
   int r = idx / half, t = idx - r * half;
-  double f = freq[t];
-  float sz, cz, st, ct;
-  sincos_reduced((double)scale * (double)noise[r] * f, &sz, &cz);
-  sincos_reduced((double)scale * (double)tau * f, &st, &ct);
-  feat[(size_t)r * d + t] = from_f<TA>(cz + ct);
-  feat[(size_t)r * d + half + t] = from_f<TA>(sz + st);
+  float sz, cz;
+  sincos_reduced((double)scale * (double)noise[r] * freq[t], &sz, &cz);
+  feat[(size_t)r * d + t] = from_f<TA>(cz + tau_feat[t]);
+  feat[(size_t)r * d + half + t] = from_f<TA>(sz + tau_feat[half + t]);
 }
 
-void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, float tau,
+void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, const float* tau_feat,
                        float scale, int d, void* feat, cudaStream_t s) {
   if (n == 0) return;
   int tot = n * (d / 2);
   if (bf16)
-    kf_launch(k_noise_feat<__nv_bfloat16>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau, scale, d,
-                                                                   (__nv_bfloat16*)feat);
+    kf_launch(k_noise_feat<__nv_bfloat16>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau_feat,
+              scale, d, (__nv_bfloat16*)feat);
   else
-    kf_launch(k_noise_feat<float>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau, scale, d,
-                                                           (float*)feat);
+    kf_launch(k_noise_feat<float>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau_feat, scale, d,
+              (float*)feat);
 }
 
 // --------------------------------------------------------------- RMSNorm

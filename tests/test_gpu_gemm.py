@@ -18,8 +18,9 @@ SHAPES = [
     (256, 30720, 768),   # LM-head shape (vocab padded to 256)
     (1000, 200, 128),    # N not a multiple of the tile
     (200, 640, 320),     # odd number of 64-wide K blocks: a short last pipeline stage
-    (4096, 768, 3072),   # OWT batch 512 k=4 MLP-down: one wave of 96 256-wide tiles
-    (3900, 700, 768),    # one wave of 256-wide tiles with ragged M and N
+    (4096, 768, 3072),   # OWT batch 512 k=4 MLP-down: one wave of 128 192-wide tiles
+    (3900, 700, 768),    # 192-wide tiles with ragged M and N (the last W box partly past N)
+    (4096, 768, 768),    # OWT batch 512 k=4 O projection: 192-wide tiles
     (2100, 2340, 768),   # persistent 256-wide tiles with ragged M and N
     (4096, 2304, 768),   # OWT batch 512 k=4 QKV shape: two tiles per CTA
     (4096, 3072, 768),   # OWT batch 512 k=4 MLP-up shape: 384 tiles on the persistent loop
