@@ -556,9 +556,10 @@ def run_serving(args):
 
 def run_train_attention(args):
     """SingleForward / DoubleForward attention (App. C.2), bf16, head_dim 64:
-    the mask-aware kernel against the same kernel visiting every key tile
-    (the dense-mask cost).  Reports TFLOP/s over the mask's pairs
-    (4 * 64 flops per visible (query, key) pair)."""
+    the mask-aware tcgen05 kernel, against the same kernel visiting every
+    key tile (the dense-mask cost) and against the warp-level MMA kernel.
+    Reports TFLOP/s over the mask's pairs (4 * 64 flops per visible
+    (query, key) pair)."""
     import ctypes
     import torch
     from paper_2606_10820_gb300 import build as kbuild
@@ -581,7 +582,7 @@ def run_train_attention(args):
             pairs += k * ctx + N * k * k + N * k * (k + 1) // 2
         flops = 4.0 * 64 * pairs * B * H
         res = {}
-        for dense in (0, 1):
+        for dense in (0, 1, 2):     # tcgen05, tcgen05 every key tile, warp-level MMA
             def call():
                 lib.kf_op_train_attention(blocks, B, H, N, k, 0, T, q.data_ptr(), kk.data_ptr(),
                                           v.data_ptr(), out.data_ptr(), dense, None)
@@ -599,6 +600,7 @@ def run_train_attention(args):
         print(json.dumps({
             "metric": "training attention (App. C.2) TFLOP/s over the mask's pairs", "unit": "TFLOP/s",
             "value": tf, "ms": res[0], "dense_mask_ms": res[1], "speedup_vs_dense_mask": res[1] / res[0],
+            "warp_mma_ms": res[2], "speedup_vs_warp_mma": res[2] / res[0],
             "roofline": {"bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": tf / pk["bf16_tflops"], "peak_source": peak_src},
             "config": {"mask": "SingleForward" if blocks == 1 else "DoubleForward", "batch": B, "heads": H,

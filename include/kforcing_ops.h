@@ -114,12 +114,19 @@ int kf_op_status(void* stream);
  * Future-2 alone, reusing the other rows' keys).  out: [B][q_end - q_begin][H][64]
  * fp32, device, caller-owned.  Scale 1/sqrt(64), fp32 softmax, probabilities
  * rounded to bf16 for the P.V product.
- * dense = 0 visits only the key tiles a query tile can see (the context prefix
- * and its windows: O(k) pairs relative to AR attention); dense = 1 visits every
- * key tile with the same mask (the cost of a dense mask, for comparison).
- * Errors: KF_E_ARG (sizes, ranges, alignment), KF_E_CUDA.  Asynchronous on
- * `stream` (NULL: the default stream).
+ * dense: flags.  Without KF_TRAIN_ATTN_DENSE only the key tiles a query tile
+ * can see are visited (the context prefix and its windows: O(k) pairs
+ * relative to AR attention); with it every key tile, with the same mask (the
+ * cost of a dense mask, for comparison).  The kernel runs on tcgen05 (S and
+ * O in tensor memory, 128 query rows and 128-key tiles per step);
+ * KF_TRAIN_ATTN_WARP_MMA selects the warp-level MMA kernel instead (64 query
+ * rows, 64-key tiles), for comparison.
+ * Errors: KF_E_ARG (sizes, ranges, alignment, unknown flags), KF_E_CUDA.
+ * Asynchronous on `stream` (NULL: the default stream); a bounded wait that
+ * ran out inside the tcgen05 kernel is reported by kf_op_status (KF_E_DEVICE).
  */
+#define KF_TRAIN_ATTN_DENSE 1
+#define KF_TRAIN_ATTN_WARP_MMA 2
 int kf_op_train_attention(int32_t blocks, int32_t B, int32_t H, int32_t N, int32_t k,
                           int32_t q_begin, int32_t q_end, const void* q, const void* kk,
                           const void* v, float* out, int32_t dense, void* stream);

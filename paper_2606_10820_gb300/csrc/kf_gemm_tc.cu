@@ -748,6 +748,26 @@ bool encode_rows_map_bf16(CUtensorMap* m, const void* base, uint64_t rows, int c
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_map_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims, const uint64_t* strides,
+                     const uint32_t* box) {
+  if (!get_encode() || rank < 1 || rank > 5 || (reinterpret_cast<uintptr_t>(base) & 15) || box[0] * 2 > 128)
+    return false;
+  cuuint64_t d[5], st[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+    if (i > 0) {
+      if (strides[i - 1] % 16) return false;
+      st[i - 1] = strides[i - 1];
+    }
+  }
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, st, bx, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool tc_gemm_supported(const GemmDesc& g) {
   if (g.K % kBK || g.K == 0 || g.M <= 0 || g.N <= 0) return false;
   if ((g.lda * 2) % 16 || (g.ldw * 2) % 16) return false;

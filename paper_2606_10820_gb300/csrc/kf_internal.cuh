@@ -472,6 +472,10 @@ bool attention_mma_supported(bool bf16, int hd, int rows);
 int launch_attention_mma(const AttnArgs& a, int n_groups, int rows, int max_keys, cudaStream_t s,
                          bool* merged);
 
+// the op entry points' error word on the current device, cleared on s
+// (read back by kf_op_status); nullptr on failure
+int* op_error_word(cudaStream_t s);
+
 // message for kf_last_error(NULL) (calls without a context)
 void set_global_error(const std::string& msg);
 

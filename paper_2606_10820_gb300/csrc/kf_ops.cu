@@ -42,6 +42,23 @@ int ensure_err(int dev) {
 }
 }  // namespace
 
+namespace kf {
+// the calling thread's device's op error word, cleared on `s` (kf_op_status
+// reads it); nullptr if it cannot be had
+int* op_error_word(cudaStream_t s) {
+  int dev = 0;
+  if (current_device(&dev) != KF_OK) return nullptr;
+  int* err = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_ops_mu);
+    if (ensure_err(dev) != KF_OK) return nullptr;
+    err = g_ops[dev].err;
+  }
+  if (cudaMemsetAsync(err, 0, sizeof(int), s) != cudaSuccess) return nullptr;
+  return err;
+}
+}  // namespace kf
+
 // the LM-head GEMM with the chunk-record epilogue, then the token select
 static int head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const void* w_head,
                        const float* noise, float tau, int32_t map_kind, int32_t* tokens,

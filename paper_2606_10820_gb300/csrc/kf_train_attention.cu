@@ -31,6 +31,7 @@
 #include "../../include/kforcing_ops.h"
 #include "kf_internal.cuh"
 #include "kf_mma.cuh"
+#include "kf_tc.cuh"
 
 namespace kf {
 namespace {
@@ -287,6 +288,341 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
   }
 }
 
+// ------------------------------------------------------------------ tcgen05
+// The same attention on the 5th-generation tensor cores.  A CTA takes 128
+// query rows of one (sequence, head) and walks the same key ranges in tiles
+// of 128 keys (each range's tiles start at its first key; keys past the
+// range's end are masked, so no key is counted twice):
+//   warp 0      TMA: Q once, then K and V tiles of [128 keys][64] bf16
+//               (128-byte swizzle) into a two-stage ring;
+//   warp 1      one thread issues tcgen05.mma: S_j = Q K_j^T (M = 128 rows,
+//               N = 128 keys, K = 64) into one of two TMEM buffers, and
+//               O_j = P_j V_j (M = 128, N = 64, K = 128 keys; V is the
+//               MN-major operand as loaded) into one of two more;
+//   warps 2..9  two threads per query row (TMEM lane), each with half of
+//               its keys and of its output (four threads measured 5 % slower:
+//               the per-tile chain of waits and barriers, not the arithmetic,
+//               bounds the softmax): mask S_j, share the row max
+//               through shared memory, keep the running max m and their part
+//               of the sum l, write P_j = exp2(S_j - m) as bf16 into shared
+//               memory (K-major, swizzled: the A operand of P V) and fold
+//               O_j into their fp32 output dims, o <- o exp2(m_prev - m) + O_j.
+// S of tile j + 1 is computed while the softmax works on tile j.  Every
+// wait is bounded; a wait that runs out sets the error word and ends the
+// CTA's loops.
+namespace {
+constexpr int kTcRows = 128;
+constexpr int kTcKeys = 128;
+constexpr int kTcSplit = 2;                          // softmax threads per query row
+constexpr int kTcSoftmax = 128 * kTcSplit;           // kTcSplit warps per TMEM lane quarter
+constexpr int kTcThreads = 64 + kTcSoftmax;
+constexpr int kTcPart = kTcKeys / kTcSplit;          // keys of a row per softmax thread
+constexpr int kTcOut = kHD / kTcSplit;               // output dims of a row per softmax thread
+constexpr uint32_t kTcTile = kTcRows * kHD * 2;       // 16 KB: Q, a K tile, a V tile
+constexpr uint32_t kTcP = kTcRows * kTcKeys * 2;      // 32 KB: one P tile (two 64-key atoms)
+// [Q][K 2][V 2][P 2], the barriers and shared scalars (256 B), then the
+// row-max exchange [2 tiles][kTcSplit parts][128 rows] and the row sums
+// [kTcSplit][128]
+constexpr size_t tc_smem_bytes() {
+  return 1024 + 5 * (size_t)kTcTile + 2 * (size_t)kTcP + 256 + 3 * kTcSplit * 128 * 4;
+}
+}  // namespace
+
+// AND of `ok` over the softmax threads (named barrier 1): every one of
+// them takes the same path after a bounded wait
+__device__ __forceinline__ bool softmax_all(bool ok) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.and.pred p, 1, %2, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)ok), "n"(kTcSoftmax)
+      : "memory");
+  return r != 0;
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+                     const __grid_constant__ CUtensorMap map_v, TrainAttnArgs a, int* d_err) {
+  pdl_trigger();
+  extern __shared__ __align__(1024) uint8_t tsm_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tsm_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t sQ = smem_u32(sm);
+  const uint32_t sK = sQ + kTcTile;                  // [2]
+  const uint32_t sV = sK + 2 * kTcTile;              // [2]
+  uint8_t* Pp = sm + 5 * kTcTile;                    // [2][2 atoms][128 rows][128 B]
+  const uint32_t sP = smem_u32(Pp);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + 5 * kTcTile + 2 * kTcP);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;       // [2]
+  uint64_t* kv_empty = bars + 3;      // [2]
+  uint64_t* s_full = bars + 5;        // [2]
+  uint64_t* p_full = bars + 7;        // [2]: P_j written (and S_j read)
+  uint64_t* o_full = bars + 9;        // [2]
+  uint64_t* o_empty = bars + 11;      // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 13);
+  int* s_rng = reinterpret_cast<int*>(tmem_slot + 1);   // cmax, w1lo, w1hi, w2lo, w2hi, cmin
+  int* s_cnt = s_rng + 6;                                // tiles whose K/V the MMA has taken
+  float* s_mx = reinterpret_cast<float*>(sm + 5 * kTcTile + 2 * kTcP + 256);   // [2][2][128]
+  float* s_l = s_mx + 2 * kTcSplit * kTcRows;                                  // [kTcSplit][128]
+
+  const int q0 = a.q_begin + blockIdx.x * kTcRows, h = blockIdx.y, b = blockIdx.z;
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int quarter = warp & 3;                 // softmax warps: TMEM lanes 32 quarter ..
+  const int row = 32 * quarter + lane;          // this softmax thread's query row in the tile
+  const int part = (warp - 2) >> 2;             // its keys kTcPart part .. and output dims kTcOut part ..
+  RowVis v{-1, 0, 0, 0, 0};
+  if (warp >= 2) v = row_vis(a, q0 + row);
+
+  if (t == 0) {
+    mbar_init(smem_u32(q_full), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&kv_full[i]), 1);
+      mbar_init(smem_u32(&kv_empty[i]), 1);
+      mbar_init(smem_u32(&s_full[i]), 1);
+      mbar_init(smem_u32(&p_full[i]), 1);
+      mbar_init(smem_u32(&o_full[i]), 1);
+      mbar_init(smem_u32(&o_empty[i]), 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_q)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_k)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_v)) : "memory");
+    s_rng[0] = -1; s_rng[1] = 1 << 30; s_rng[2] = 0; s_rng[3] = 1 << 30; s_rng[4] = 0; s_rng[5] = 1 << 30;
+    s_cnt[0] = 0;
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(512)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  const uint32_t tmem = *tmem_slot;
+  // the key ranges of the CTA's rows (their union), and the context keys
+  // every valid row sees
+  if (warp >= 2 && v.ctx >= 0) {
+    atomicMax(&s_rng[0], v.ctx);
+    atomicMin(&s_rng[5], v.ctx);
+    if (v.w1hi > v.w1lo) { atomicMin(&s_rng[1], v.w1lo); atomicMax(&s_rng[2], v.w1hi); }
+    if (v.w2hi > v.w2lo) { atomicMin(&s_rng[3], v.w2lo); atomicMax(&s_rng[4], v.w2hi); }
+  }
+  __syncthreads();
+  int rlo[3], rhi[3], nr = 0;
+  if (a.dense) {
+    rlo[0] = 0; rhi[0] = a.T; nr = 1;
+  } else {
+    if (s_rng[0] >= 0) { rlo[nr] = 0; rhi[nr] = s_rng[0] + 1; ++nr; }
+    if (s_rng[2] > s_rng[1]) { rlo[nr] = s_rng[1]; rhi[nr] = s_rng[2]; ++nr; }
+    if (s_rng[4] > s_rng[3]) { rlo[nr] = s_rng[3]; rhi[nr] = s_rng[4]; ++nr; }
+  }
+  const int cmin = s_rng[5];
+  int n_tiles = 0;
+  for (int i = 0; i < nr; ++i) n_tiles += ceil_div(rhi[i] - rlo[i], kTcKeys);
+  auto tile_at = [&](int j, int* lo, int* hi) {
+    for (int i = 0; i < nr; ++i) {
+      const int n = ceil_div(rhi[i] - rlo[i], kTcKeys);
+      if (j < n) { *lo = rlo[i] + j * kTcKeys; *hi = rhi[i]; return; }
+      j -= n;
+    }
+    *lo = 0; *hi = 0;
+  };
+  pdl_wait();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_expect_tx(smem_u32(q_full), kTcTile);
+      tma_load_4d(sQ, &map_q, smem_u32(q_full), 0, h, q0, b);
+      int issued = 0;
+      bool ok = true;
+      for (int j = 0; j < n_tiles; ++j) {
+        const int st = j & 1;
+        if (j >= 2 && !mbar_wait(smem_u32(&kv_empty[st]), ((j - 2) >> 1) & 1, d_err)) { ok = false; break; }
+        int kt, kend;
+        tile_at(j, &kt, &kend);
+        mbar_expect_tx(smem_u32(&kv_full[st]), 2 * kTcTile);
+        tma_load_4d(sK + st * kTcTile, &map_k, smem_u32(&kv_full[st]), 0, h, kt, b);
+        tma_load_4d(sV + st * kTcTile, &map_v, smem_u32(&kv_full[st]), 0, h, kt, b);
+        issued = j + 1;
+      }
+      if (!ok) {
+        // let the copies still in flight land before the CTA ends (bounded)
+        for (int j = *(volatile int*)s_cnt; j < issued; ++j)
+          mbar_wait(smem_u32(&kv_full[j & 1]), (j >> 1) & 1, d_err);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(kTcRows, kTcKeys);
+      constexpr uint32_t idesc_o = idesc_bf16(kTcRows, kHD) | (1u << 16);   // B (V) MN-major
+      bool ok = mbar_wait(smem_u32(q_full), 0, d_err);
+      // O_i = P_i V_i into TMEM columns 256 + 64 (i % 2)
+      auto issue_pv = [&](int i) -> bool {
+        const int st = i & 1;
+        if (!mbar_wait(smem_u32(&p_full[st]), (i >> 1) & 1, d_err)) return false;
+        if (i >= 2 && !mbar_wait(smem_u32(&o_empty[st]), ((i - 2) >> 1) & 1, d_err)) return false;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t pa = sP + st * kTcP, vb = sV + st * kTcTile;
+#pragma unroll
+        for (int kk = 0; kk < kTcKeys / 16; ++kk)
+          mma_bf16(tmem + 256 + 64 * st, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
+                   sdesc_mn(vb + kk * 16 * 128), idesc_o, kk > 0 ? 1u : 0u);
+        mma_commit(smem_u32(&o_full[st]));
+        mma_commit(smem_u32(&kv_empty[st]));
+        return true;
+      };
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int st = j & 1;
+        if (!mbar_wait(smem_u32(&kv_full[st]), (j >> 1) & 1, d_err)) { ok = false; break; }
+        *(volatile int*)s_cnt = j + 1;
+        // S buffer st is free once the softmax has read S_{j-2}
+        if (j >= 2 && !mbar_wait(smem_u32(&p_full[st]), ((j - 2) >> 1) & 1, d_err)) { ok = false; break; }
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        const uint32_t kb = sK + st * kTcTile;
+#pragma unroll
+        for (int kk = 0; kk < kHD / 16; ++kk)
+          mma_bf16(tmem + kTcKeys * st, sdesc(sQ + kk * 32), sdesc(kb + kk * 32), idesc_s, kk > 0 ? 1u : 0u);
+        mma_commit(smem_u32(&s_full[st]));
+        if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+      }
+      if (ok && n_tiles > 0) issue_pv(n_tiles - 1);
+    }
+    __syncwarp();
+  } else {
+    // softmax: kTcSplit threads per query row, `part` of its keys and output each
+    static_assert(kTcPart % 32 == 0 && kTcPart <= 64 && (kTcOut == 16 || kTcOut == 32),
+                  "32-column TMEM loads of S, one load of O per thread");
+    const float sc = 1.4426950408889634f * rsqrtf((float)kHD);
+    const uint32_t lane_base = (uint32_t)(32 * quarter) << 16;
+    const int kb0 = kTcPart * part;               // first key of this thread's part of a tile
+    float m = -INFINITY, l = 0.f, alpha_prev = 1.f;
+    float o[kTcOut];
+#pragma unroll
+    for (int d = 0; d < kTcOut; ++d) o[d] = 0.f;
+    // this row's 16-byte chunks of P buffer 0 for keys kb0 .. kb0 + 31: atom
+    // kb0 / 64, chunks (kb0 % 64) / 8 + q at position chunk ^ (row % 8)
+    const uint32_t prow = sP + (kb0 >> 6) * (kTcP / 2) + row * 128;
+    const int chunk0 = (kb0 & 63) >> 3;
+    bool ok = true;
+    // the visible keys kb0 + i (i < kTcPart) of a row as a bit mask: [lo, hi) relative to the tile
+    auto range_bits = [&](int lo, int hi) -> unsigned long long {
+      lo = max(lo - kb0, 0);
+      hi = min(hi - kb0, kTcPart);
+      if (hi <= lo) return 0ull;
+      const unsigned long long up = hi >= 64 ? ~0ull : ((1ull << hi) - 1ull);
+      return up & ~((1ull << lo) - 1ull);
+    };
+    // o <- o * alpha + O_i (this thread's output dims of P_i V_i), then free
+    // its TMEM buffer
+    auto fold_o = [&](int i, float alpha) -> bool {
+      const int st = i & 1;
+      if (!softmax_all(mbar_wait(smem_u32(&o_full[st]), (i >> 1) & 1, d_err))) return false;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      float r[kTcOut];
+      if constexpr (kTcOut == 32) tmem_ld32(tmem + lane_base + 256 + 64 * st + kTcOut * part, r);
+      else tmem_ld16(tmem + lane_base + 256 + 64 * st + kTcOut * part, r);
+#pragma unroll
+      for (int d = 0; d < kTcOut; ++d) o[d] = o[d] * alpha + r[d];
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&o_empty[st])) : "memory");
+      return true;
+    };
+    for (int j = 0; j < n_tiles; ++j) {
+      const int st = j & 1;
+      int kt, kend;
+      tile_at(j, &kt, &kend);
+      // visible keys of this part: the context prefix [0, ctx], the windows,
+      // none past the range's end (each key belongs to one range's tiles)
+      const int lim = min(kend - kt, kTcKeys);
+      const bool open = !a.dense && kt + kTcKeys - 1 < kend && kt + kTcKeys - 1 <= cmin && v.ctx >= 0;
+      unsigned long long vis = ~0ull;
+      if (!open)
+        vis = (range_bits(0, v.ctx - kt + 1) | range_bits(v.w1lo - kt, v.w1hi - kt) |
+               range_bits(v.w2lo - kt, v.w2hi - kt)) &
+              range_bits(0, lim);
+      if (!softmax_all(mbar_wait(smem_u32(&s_full[st]), (j >> 1) & 1, d_err))) { ok = false; break; }
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      float sv[kTcPart];
+#pragma unroll
+      for (int c = 0; c < kTcPart / 32; ++c) tmem_ld32(tmem + lane_base + kTcKeys * st + kb0 + 32 * c, sv + 32 * c);
+      // raw scores: sc > 0, so the max commutes with the scaling
+      float mx = -INFINITY;
+#pragma unroll
+      for (int e = 0; e < kTcPart; ++e) {
+        sv[e] = ((vis >> e) & 1ull) ? sv[e] : -INFINITY;
+        mx = fmaxf(mx, sv[e]);
+      }
+      // the row's max over its parts
+      s_mx[(st * kTcSplit + part) * kTcRows + row] = mx;
+      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      mx = s_mx[(st * kTcSplit) * kTcRows + row];
+#pragma unroll
+      for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
+      const float mn = fmaxf(m, mx * sc);
+      const float alpha = (mn == -INFINITY) ? 1.f : ex2(m - mn);
+      // P = exp2(S sc - mn) rounded to bf16 (ex2(-inf) = 0 for masked keys),
+      // the sum of the rounded values
+      const uint32_t pbase = prow + st * kTcP;
+      const float nmn = mn == -INFINITY ? 0.f : -mn;
+      float ps = 0.f;
+#pragma unroll
+      for (int q = 0; q < kTcPart / 8; ++q) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int e = 8 * q + 2 * u;
+          pk[u] = pack_bf16(ex2(fmaf(sv[e], sc, nmn)), ex2(fmaf(sv[e + 1], sc, nmn)));
+          const float2 f = unpack_bf16(pk[u]);
+          ps += f.x + f.y;
+        }
+        const uint32_t addr = pbase + (((chunk0 + q) ^ (row & 7)) << 4);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
+                     "r"(pk[3])
+                     : "memory");
+      }
+      m = mn;
+      l = l * alpha + ps;
+      // S_j read, P_j written: to the tensor cores (async proxy)
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
+      // O_{j-1} (relative to the max before this tile) into the output
+      if (j >= 1 && !fold_o(j - 1, alpha_prev)) { ok = false; break; }
+      alpha_prev = alpha;
+    }
+    if (ok && n_tiles > 0) ok = fold_o(n_tiles - 1, alpha_prev);
+    if (ok) {
+      // the row's sum over its parts, in a fixed order
+      s_l[part * kTcRows + row] = l;
+      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      float lt = 0.f;
+#pragma unroll
+      for (int q = 0; q < kTcSplit; ++q) lt += s_l[q * kTcRows + row];
+      const int qi = q0 + row;
+      if (qi < a.q_end && lt > 0.f) {
+        const float inv = 1.f / lt;
+        float* dst =
+            a.out + (((size_t)b * (a.q_end - a.q_begin) + (qi - a.q_begin)) * a.H + h) * kHD + kTcOut * part;
+#pragma unroll
+        for (int d = 0; d < kTcOut; d += 4)
+          *reinterpret_cast<float4*>(dst + d) = make_float4(o[d] * inv, o[d + 1] * inv, o[d + 2] * inv, o[d + 3] * inv);
+      }
+    }
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+}
+
 }  // namespace kf
 
 using namespace kf;
@@ -301,12 +637,32 @@ extern "C" int kf_op_train_attention(int32_t blocks, int32_t B, int32_t H, int32
   if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(kk) | reinterpret_cast<uintptr_t>(v) |
        reinterpret_cast<uintptr_t>(out)) & 15)
     return KF_E_ARG;
+  if (dense & ~(KF_TRAIN_ATTN_DENSE | KF_TRAIN_ATTN_WARP_MMA)) return KF_E_ARG;
   TrainAttnArgs a{static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(kk),
                   static_cast<const __nv_bfloat16*>(v), out, N, k, blocks, (int)T, H, q_begin, q_end,
-                  dense ? 1 : 0};
-  static PerDevice attr;
-  set_smem_attr(attr, k_train_attention, smem_bytes());
-  const dim3 grid(ceil_div(q_end - q_begin, kRows), H, B);
-  kf_launch(k_train_attention, grid, dim3(kThr), smem_bytes(), (cudaStream_t)stream, a);
+                  (dense & KF_TRAIN_ATTN_DENSE) ? 1 : 0};
+  cudaStream_t s = (cudaStream_t)stream;
+  if (dense & KF_TRAIN_ATTN_WARP_MMA) {
+    static PerDevice attr;
+    set_smem_attr(attr, k_train_attention, smem_bytes());
+    const dim3 grid(ceil_div(q_end - q_begin, kRows), H, B);
+    kf_launch(k_train_attention, grid, dim3(kThr), smem_bytes(), s, a);
+    return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
+  }
+  // q, kk, v as [B][T][H][64] with the head one coordinate: boxes of one
+  // head's 128 consecutive tokens (rows past T read as zero)
+  const uint64_t dims[4] = {64, (uint64_t)H, (uint64_t)T, (uint64_t)B};
+  const uint64_t strides[3] = {128, (uint64_t)H * 128, (uint64_t)T * H * 128};
+  const uint32_t box[4] = {64, 1, kTcRows, 1};
+  CUtensorMap mq, mk, mv;
+  if (!encode_map_bf16(&mq, q, 4, dims, strides, box) || !encode_map_bf16(&mk, kk, 4, dims, strides, box) ||
+      !encode_map_bf16(&mv, v, 4, dims, strides, box))
+    return KF_E_CUDA;
+  int* err = op_error_word(s);
+  if (!err) return KF_E_CUDA;
+  static PerDevice attr_tc;
+  set_smem_attr(attr_tc, k_train_attention_tc, tc_smem_bytes());
+  const dim3 grid(ceil_div(q_end - q_begin, kTcRows), H, B);
+  kf_launch(k_train_attention_tc, grid, dim3(kTcThreads), tc_smem_bytes(), s, mq, mk, mv, a, err);
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
 }

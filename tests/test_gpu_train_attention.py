@@ -59,8 +59,9 @@ CASES = [
 ]
 
 
+# flags: 1 every key tile (dense mask), 2 the warp-level MMA kernel instead of tcgen05
 @pytest.mark.parametrize("blocks,B,H,N,k", CASES)
-@pytest.mark.parametrize("dense", [0, 1])
+@pytest.mark.parametrize("dense", [0, 1, 2, 3])
 def test_train_attention_matches_dense_oracle(env, blocks, B, H, N, k, dense):
     torch, lib = env
     q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, dense=dense, seed=N * 31 + k)
@@ -77,15 +78,34 @@ def test_double_future2_only_rows(env):
     _check(q, kk, v, out, blocks, N, k, qb, qe)
 
 
-def test_long_sequence_sampled_rows(env):
+@pytest.mark.parametrize("flags", [0, 2])
+def test_long_sequence_sampled_rows(env, flags):
     """N = 512, k = 4 (T = 2560): rows sampled across the blocks."""
     torch, lib = env
     blocks, B, H, N, k = 1, 1, 2, 512, 4
-    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, seed=9)
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, dense=flags, seed=9)
     mask = ta.mask_single(N, k)
     rows = np.array([0, 1, 127, 128, 511, N, N + 3, N + 4 * 200 + 2, N + 4 * 511 + 3])
     ref = ta.masked_attention(q[0, rows], kk[0], v[0], mask[rows])
     assert np.abs(out[0, rows] - ref).max() <= 8e-3 * np.abs(v[0]).max()
+
+
+def test_kernels_agree_double_forward(env):
+    """DoubleForward N = 300, k = 4 (T = 2700, ragged 128-row tiles): the
+    tcgen05 kernel and the warp-level MMA kernel within the tolerance of each
+    other on every row, and the oracle on sampled rows."""
+    torch, lib = env
+    blocks, B, H, N, k = 2, 2, 3, 300, 4
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, dense=0, seed=11)
+    out2 = _run(torch, lib, blocks, B, H, N, k, dense=2, seed=11)[3]
+    assert np.isfinite(out).all()
+    assert np.abs(out - out2).max() <= 8e-3 * np.abs(v).max()
+    mask = ta.mask_full(N, k, blocks)
+    rows = np.array([0, 127, 128, 299, N, N + 517, N + N * k - 1, N + N * k, N + N * k + 3 * 77 + 2,
+                     N + 2 * N * k - 1])
+    for b in range(B):
+        ref = ta.masked_attention(q[b, rows], kk[b], v[b], mask[rows])
+        assert np.abs(out[b, rows] - ref).max() <= 8e-3 * np.abs(v[b]).max()
 
 
 def test_argument_errors(env):
@@ -96,3 +116,5 @@ def test_argument_errors(env):
     for args in [(3, 1, 1, 4, 2, 0, 12), (1, 1, 1, 4, 2, 0, 13), (1, 1, 1, 4, 2, 5, 5),
                  (1, 0, 1, 4, 2, 0, 12), (2, 1, 1, 4, 0, 0, 4)]:
         assert lib.kf_op_train_attention(*args, p, p, p, out.data_ptr(), 0, None) == -1, args
+    # an unknown flag
+    assert lib.kf_op_train_attention(1, 1, 1, 4, 2, 0, 12, p, p, p, out.data_ptr(), 4, None) == -1
