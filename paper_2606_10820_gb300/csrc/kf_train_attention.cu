@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
 // of 128 keys (each range's tiles start at its first key; keys past the
 // range's end are masked, so no key is counted twice):
 //   warp 0      TMA: Q once, then K and V tiles of [128 keys][64] bf16
-//               (128-byte swizzle) into a two-stage ring;
+//               (128-byte swizzle) into a four-stage ring;
 //   warp 1      one thread issues tcgen05.mma: S_j = Q K_j^T (M = 128 rows,
 //               N = 128 keys, K = 64) into one of two TMEM buffers, and
 //               O_j = P_j V_j (M = 128, N = 64, K = 128 keys; V is the
@@ -320,11 +320,15 @@ constexpr int kTcPart = kTcKeys / kTcSplit;          // keys of a row per softma
 constexpr int kTcOut = kHD / kTcSplit;               // output dims of a row per softmax thread
 constexpr uint32_t kTcTile = kTcRows * kHD * 2;       // 16 KB: Q, a K tile, a V tile
 constexpr uint32_t kTcP = kTcRows * kTcKeys * 2;      // 32 KB: one P tile (two 64-key atoms)
-// [Q][K 2][V 2][P 2], the barriers and shared scalars (256 B), then the
-// row-max exchange [2 tiles][kTcSplit parts][128 rows] and the row sums
-// [kTcSplit][128]
+// K/V ring stages: tile j's copies are issued while tile j - 1 is in the
+// softmax and tile j - 2's V still feeds P V (two stages measured 2.0 us per
+// tile, the copy latency on the critical path)
+constexpr int kTcStages = 4;
+// [Q][K stages][V stages][P 2], the barriers and shared scalars (256 B),
+// then the row-max exchange [2 tiles][kTcSplit parts][128 rows] and the row
+// sums [kTcSplit][128]
 constexpr size_t tc_smem_bytes() {
-  return 1024 + 5 * (size_t)kTcTile + 2 * (size_t)kTcP + 256 + 3 * kTcSplit * 128 * 4;
+  return 1024 + (1 + 2 * kTcStages) * (size_t)kTcTile + 2 * (size_t)kTcP + 256 + 3 * kTcSplit * 128 * 4;
 }
 }  // namespace
 
@@ -350,22 +354,23 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
   extern __shared__ __align__(1024) uint8_t tsm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tsm_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(sm);
-  const uint32_t sK = sQ + kTcTile;                  // [2]
-  const uint32_t sV = sK + 2 * kTcTile;              // [2]
-  uint8_t* Pp = sm + 5 * kTcTile;                    // [2][2 atoms][128 rows][128 B]
+  const uint32_t sK = sQ + kTcTile;                  // [kTcStages]
+  const uint32_t sV = sK + kTcStages * kTcTile;      // [kTcStages]
+  constexpr uint32_t kPOff = (1 + 2 * kTcStages) * kTcTile;
+  uint8_t* Pp = sm + kPOff;                          // [2][2 atoms][128 rows][128 B]
   const uint32_t sP = smem_u32(Pp);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + 5 * kTcTile + 2 * kTcP);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kPOff + 2 * kTcP);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;       // [2]
-  uint64_t* kv_empty = bars + 3;      // [2]
-  uint64_t* s_full = bars + 5;        // [2]
-  uint64_t* p_full = bars + 7;        // [2]: P_j written (and S_j read)
-  uint64_t* o_full = bars + 9;        // [2]
-  uint64_t* o_empty = bars + 11;      // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 13);
+  uint64_t* kv_full = bars + 1;                      // [kTcStages]
+  uint64_t* kv_empty = kv_full + kTcStages;          // [kTcStages]
+  uint64_t* s_full = kv_empty + kTcStages;           // [2]
+  uint64_t* p_full = s_full + 2;                     // [2]: P_j written (and S_j read)
+  uint64_t* o_full = p_full + 2;                     // [2]
+  uint64_t* o_empty = o_full + 2;                    // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_empty + 2);
   int* s_rng = reinterpret_cast<int*>(tmem_slot + 1);   // cmax, w1lo, w1hi, w2lo, w2hi, cmin
   int* s_cnt = s_rng + 6;                                // tiles whose K/V the MMA has taken
-  float* s_mx = reinterpret_cast<float*>(sm + 5 * kTcTile + 2 * kTcP + 256);   // [2][2][128]
+  float* s_mx = reinterpret_cast<float*>(sm + kPOff + 2 * kTcP + 256);         // [2][kTcSplit][128]
   float* s_l = s_mx + 2 * kTcSplit * kTcRows;                                  // [kTcSplit][128]
 
   const int q0 = a.q_begin + blockIdx.x * kTcRows, h = blockIdx.y, b = blockIdx.z;
@@ -378,9 +383,11 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
 
   if (t == 0) {
     mbar_init(smem_u32(q_full), 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kTcStages; ++i) {
       mbar_init(smem_u32(&kv_full[i]), 1);
       mbar_init(smem_u32(&kv_empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
       mbar_init(smem_u32(&p_full[i]), 1);
       mbar_init(smem_u32(&o_full[i]), 1);
@@ -440,8 +447,11 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       int issued = 0;
       bool ok = true;
       for (int j = 0; j < n_tiles; ++j) {
-        const int st = j & 1;
-        if (j >= 2 && !mbar_wait(smem_u32(&kv_empty[st]), ((j - 2) >> 1) & 1, d_err)) { ok = false; break; }
+        const int st = j % kTcStages;
+        if (j >= kTcStages && !mbar_wait(smem_u32(&kv_empty[st]), ((j / kTcStages) - 1) & 1, d_err)) {
+          ok = false;
+          break;
+        }
         int kt, kend;
         tile_at(j, &kt, &kend);
         mbar_expect_tx(smem_u32(&kv_full[st]), 2 * kTcTile);
@@ -452,7 +462,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       if (!ok) {
         // let the copies still in flight land before the CTA ends (bounded)
         for (int j = *(volatile int*)s_cnt; j < issued; ++j)
-          mbar_wait(smem_u32(&kv_full[j & 1]), (j >> 1) & 1, d_err);
+          mbar_wait(smem_u32(&kv_full[j % kTcStages]), (j / kTcStages) & 1, d_err);
       }
     }
     __syncwarp();
@@ -467,23 +477,24 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
         if (!mbar_wait(smem_u32(&p_full[st]), (i >> 1) & 1, d_err)) return false;
         if (i >= 2 && !mbar_wait(smem_u32(&o_empty[st]), ((i - 2) >> 1) & 1, d_err)) return false;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t pa = sP + st * kTcP, vb = sV + st * kTcTile;
+        const int kvs = i % kTcStages;
+        const uint32_t pa = sP + st * kTcP, vb = sV + kvs * kTcTile;
 #pragma unroll
         for (int kk = 0; kk < kTcKeys / 16; ++kk)
           mma_bf16(tmem + 256 + 64 * st, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
                    sdesc_mn(vb + kk * 16 * 128), idesc_o, kk > 0 ? 1u : 0u);
         mma_commit(smem_u32(&o_full[st]));
-        mma_commit(smem_u32(&kv_empty[st]));
+        mma_commit(smem_u32(&kv_empty[kvs]));
         return true;
       };
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int st = j & 1;
-        if (!mbar_wait(smem_u32(&kv_full[st]), (j >> 1) & 1, d_err)) { ok = false; break; }
+        if (!mbar_wait(smem_u32(&kv_full[j % kTcStages]), (j / kTcStages) & 1, d_err)) { ok = false; break; }
         *(volatile int*)s_cnt = j + 1;
         // S buffer st is free once the softmax has read S_{j-2}
         if (j >= 2 && !mbar_wait(smem_u32(&p_full[st]), ((j - 2) >> 1) & 1, d_err)) { ok = false; break; }
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t kb = sK + st * kTcTile;
+        const uint32_t kb = sK + (j % kTcStages) * kTcTile;
 #pragma unroll
         for (int kk = 0; kk < kHD / 16; ++kk)
           mma_bf16(tmem + kTcKeys * st, sdesc(sQ + kk * 32), sdesc(kb + kk * 32), idesc_s, kk > 0 ? 1u : 0u);
