@@ -332,21 +332,6 @@ constexpr size_t tc_smem_bytes() {
 }
 }  // namespace
 
-// AND of `ok` over the softmax threads (named barrier 1): every one of
-// them takes the same path after a bounded wait
-__device__ __forceinline__ bool softmax_all(bool ok) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\t"
-      "setp.ne.u32 q, %1, 0;\n\t"
-      "bar.red.and.pred p, 1, %2, q;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(r)
-      : "r"((uint32_t)ok), "n"(kTcSoftmax)
-      : "memory");
-  return r != 0;
-}
-
 __global__ void __launch_bounds__(kTcThreads, 1)
 k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                      const __grid_constant__ CUtensorMap map_v, TrainAttnArgs a, int* d_err) {
@@ -370,6 +355,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_empty + 2);
   int* s_rng = reinterpret_cast<int*>(tmem_slot + 1);   // cmax, w1lo, w1hi, w2lo, w2hi, cmin
   int* s_cnt = s_rng + 6;                                // tiles whose K/V the MMA has taken
+  volatile int* s_abort = s_cnt + 1;                     // a softmax thread's wait ran out
   float* s_mx = reinterpret_cast<float*>(sm + kPOff + 2 * kTcP + 256);         // [2][kTcSplit][128]
   float* s_l = s_mx + 2 * kTcSplit * kTcRows;                                  // [kTcSplit][128]
 
@@ -399,6 +385,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_v)) : "memory");
     s_rng[0] = -1; s_rng[1] = 1 << 30; s_rng[2] = 0; s_rng[3] = 1 << 30; s_rng[4] = 0; s_rng[5] = 1 << 30;
     s_cnt[0] = 0;
+    *s_abort = 0;
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -528,11 +515,16 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       const unsigned long long up = hi >= 64 ? ~0ull : ((1ull << hi) - 1ull);
       return up & ~((1ull << lo) - 1ull);
     };
+    // A bounded wait that runs out raises s_abort; every softmax thread reads
+    // it after the next barrier, so all of them leave the loop together.
+    auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) {
+      if (!mbar_wait(smem_u32(bar), parity, d_err)) *s_abort = 1;
+    };
     // o <- o * alpha + O_i (this thread's output dims of P_i V_i), then free
     // its TMEM buffer
     auto fold_o = [&](int i, float alpha) -> bool {
       const int st = i & 1;
-      if (!softmax_all(mbar_wait(smem_u32(&o_full[st]), (i >> 1) & 1, d_err))) return false;
+      wait_or_abort(&o_full[st], (i >> 1) & 1);
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       float r[kTcOut];
       if constexpr (kTcOut == 32) tmem_ld32(tmem + lane_base + 256 + 64 * st + kTcOut * part, r);
@@ -541,6 +533,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       for (int d = 0; d < kTcOut; ++d) o[d] = o[d] * alpha + r[d];
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      if (*s_abort) return false;
       if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&o_empty[st])) : "memory");
       return true;
     };
@@ -557,7 +550,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
         vis = (range_bits(0, v.ctx - kt + 1) | range_bits(v.w1lo - kt, v.w1hi - kt) |
                range_bits(v.w2lo - kt, v.w2hi - kt)) &
               range_bits(0, lim);
-      if (!softmax_all(mbar_wait(smem_u32(&s_full[st]), (j >> 1) & 1, d_err))) { ok = false; break; }
+      wait_or_abort(&s_full[st], (j >> 1) & 1);
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       float sv[kTcPart];
 #pragma unroll
@@ -572,6 +565,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       // the row's max over its parts
       s_mx[(st * kTcSplit + part) * kTcRows + row] = mx;
       asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      if (*s_abort) { ok = false; break; }
       mx = s_mx[(st * kTcSplit) * kTcRows + row];
 #pragma unroll
       for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
