@@ -406,24 +406,33 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     if (v.w2hi > v.w2lo) { atomicMin(&s_rng[3], v.w2lo); atomicMax(&s_rng[4], v.w2hi); }
   }
   __syncthreads();
-  int rlo[3], rhi[3], nr = 0;
+  // the CTA's key ranges: empty ones have lo == hi (no tiles)
+  int rlo[3], rhi[3];
+  const int nr = 3;
   if (a.dense) {
-    rlo[0] = 0; rhi[0] = a.T; nr = 1;
+    rlo[0] = 0; rhi[0] = a.T;
+    rlo[1] = rhi[1] = rlo[2] = rhi[2] = 0;
   } else {
-    if (s_rng[0] >= 0) { rlo[nr] = 0; rhi[nr] = s_rng[0] + 1; ++nr; }
-    if (s_rng[2] > s_rng[1]) { rlo[nr] = s_rng[1]; rhi[nr] = s_rng[2]; ++nr; }
-    if (s_rng[4] > s_rng[3]) { rlo[nr] = s_rng[3]; rhi[nr] = s_rng[4]; ++nr; }
+    rlo[0] = 0; rhi[0] = s_rng[0] + 1;                              // 0 when no valid row
+    rlo[1] = s_rng[1]; rhi[1] = max(s_rng[1], s_rng[2]);
+    rlo[2] = s_rng[3]; rhi[2] = max(s_rng[3], s_rng[4]);
   }
   const int cmin = s_rng[5];
+  // (constant indices only: the ranges stay in registers)
   int n_tiles = 0;
-  for (int i = 0; i < nr; ++i) n_tiles += ceil_div(rhi[i] - rlo[i], kTcKeys);
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+    if (i < nr) n_tiles += ceil_div(rhi[i] - rlo[i], kTcKeys);
   auto tile_at = [&](int j, int* lo, int* hi) {
-    for (int i = 0; i < nr; ++i) {
-      const int n = ceil_div(rhi[i] - rlo[i], kTcKeys);
-      if (j < n) { *lo = rlo[i] + j * kTcKeys; *hi = rhi[i]; return; }
-      j -= n;
-    }
     *lo = 0; *hi = 0;
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+      if (i < nr) {
+        const int n = ceil_div(rhi[i] - rlo[i], kTcKeys);
+        if (j >= 0 && j < n) { *lo = rlo[i] + j * kTcKeys; *hi = rhi[i]; }
+        j -= n;
+      }
+    }
   };
   pdl_wait();
 
