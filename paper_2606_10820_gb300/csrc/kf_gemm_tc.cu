@@ -554,7 +554,9 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
   constexpr uint32_t STAGE_BYTES = A_ATOM + B_ATOM;
   constexpr uint32_t STG_BYTES = kEpiWarps * 32 * 68 * 4;
   constexpr int TMEM_COLS = tmem_alloc_cols(2 * BN);
-  static_assert(EPI != EPI_HEAD, "the LM-head records keep their two-M-tile kernel");
+  // tile order: M-tile-major (neighbouring CTAs share an A row block), or
+  // for the LM-head records N-tile-major (the M tiles of one weight tile run
+  // side by side, so each weight tile is read from HBM once)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -570,7 +572,9 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
   int* s_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tiles = ceil_div(g.N, BN), tiles = n_tiles * ceil_div(g.M, kBM);
+  const int n_tiles = ceil_div(g.N, BN), m_tiles = ceil_div(g.M, kBM), tiles = n_tiles * m_tiles;
+  auto tile_m0 = [&](int t) { return (EPI == EPI_HEAD ? t % m_tiles : t / n_tiles) * kBM; };
+  auto tile_n0 = [&](int t) { return (EPI == EPI_HEAD ? t / m_tiles : t % n_tiles) * BN; };
   const int nkb = g.K / kBK;
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -607,7 +611,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
       uint32_t stage = 0;
       bool first = true;
       for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
-        const int m0 = (t / n_tiles) * kBM, n0 = (t % n_tiles) * BN;
+        const int m0 = tile_m0(t), n0 = tile_n0(t);
         int i0 = 0;
         if (first) {
           const int pre = min(nkb, STAGES);
@@ -678,7 +682,7 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
     uint32_t ti = 0;   // epilogue warps 2 .. kEpiWarps + 1
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++ti) {
       const uint32_t buf = ti & 1;
-      const int m0 = (t / n_tiles) * kBM, n0 = (t % n_tiles) * BN;
+      const int m0 = tile_m0(t), n0 = tile_n0(t);
       // the tile's per-row data while its mainloop runs
       if (et < kBM) fill_meta<EPI>(meta, g, m0, et);
       // the first block's per-row data before the accumulator is ready
@@ -691,8 +695,19 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
       if (!s_flag[0]) break;   // timed out: the MMA warp has stopped too
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       const uint32_t lane_addr = tmem + buf * BN + ((uint32_t)(quarter * 32) << 16);
-      if (active)
+      if (EPI == EPI_HEAD) {
+        // row mode: a thread reduces its row's 32-id chunks, the two warps of
+        // a quarter alternate halves of the tile's columns
+        const int r = m0 + quarter * 32 + lane;
+#pragma unroll 1
+        for (int c = ch * (BN / 2); c < (ch + 1) * (BN / 2); c += 32) {
+          float v[32];
+          tmem_ld32(lane_addr + c, v);
+          if (r < g.M && n0 + c < g.N) epi_run32<__nv_bfloat16>(g.epi, r, n0 + c, v, g.N);
+        }
+      } else if (active) {
         epi_vec_tile<BN, EPI>(g, meta, stg + (warp - 2) * (32 * 68), lane_addr, m0, n0, quarter, ch, lane, rows);
+      }
       // every warp has read the accumulator: the MMA warp may refill it
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       epi_bar();
@@ -899,6 +914,7 @@ static int launch_persist(const GemmDesc& g, int* d_err, int num_sms, cudaStream
     case EPI_LOGITS: return launch_persist_epi<BN, STAGES, EPI_LOGITS>(g, d_err, num_sms, s);
     case EPI_STORE_F32: return launch_persist_epi<BN, STAGES, EPI_STORE_F32>(g, d_err, num_sms, s);
     case EPI_QKV: return launch_persist_epi<BN, STAGES, EPI_QKV>(g, d_err, num_sms, s);
+    case EPI_HEAD: return launch_persist_epi<BN, STAGES, EPI_HEAD>(g, d_err, num_sms, s);
   }
   return -1;
 }
@@ -922,6 +938,12 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
   // LM-head records: 256-wide tiles; above 128 rows both M tiles of a row
   // pair in one CTA (each weight tile is streamed from HBM once per 256 rows)
   if (g.epi.kind == EPI_HEAD) {
+    // above one M tile, more than a wave of 128 x 256 tiles: a persistent
+    // loop, the M tiles of each weight tile side by side (the weights are read
+    // from HBM once) and each tile's records overlapping the next tile's
+    // mainloop
+    if (g.M > kBM && !(g_gemm_flags & kGemmNoPersist) && ceil_div(g.N, 256) * ceil_div(g.M, kBM) > num_sms)
+      return launch_persist<256, 3>(g, d_err, num_sms, s);
     if (g.M > kBM) return launch_epi<256, 3, EPI_HEAD, 2, 1>(g, d_err, num_sms, s);
     return launch_epi<256, 2, EPI_HEAD, 1, 2>(g, d_err, num_sms, s);
   }
