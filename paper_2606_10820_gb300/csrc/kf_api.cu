@@ -58,8 +58,8 @@ struct kf_ctx {
   float* ne_b2 = nullptr;
   float* rope_cos = nullptr;
   float* rope_sin = nullptr;
-  double* noise_freq = nullptr;
-  float* tau_feat = nullptr;   // [d]: cos | sin of noise_scale * tau * noise_freq
+  float* noise_freq = nullptr;   // [d/2]: exp(-ln(1e4) t / (d/2)), rounded to fp32
+  float* tau_feat = nullptr;     // [d]: cos | sin of (noise_scale * tau) * noise_freq, in fp32
   // paged KV
   void* kv = nullptr;
   int n_pages = 0, max_pages = 0;
@@ -596,18 +596,21 @@ int kf_init(const kf_config* cfg_in, const kf_weights* w, void* stream, kf_ctx**
         sn[(size_t)p * half + i] = (float)std::sin(ang);
       }
     if ((r = fbuf(&c->rope_cos, cs.size())) || (r = fbuf(&c->rope_sin, sn.size()))) return bail(r);
-    std::vector<double> fr(d / 2);
-    for (int t = 0; t < d / 2; ++t) fr[t] = std::exp(-std::log(1e4) * t / (d / 2));
+    // the noise encoding's frequencies in fp32, and the temperature's
+    // encoding with the oracle's fp32 arithmetic: (scale * tau) * freq
+    std::vector<float> fr(d / 2);
+    for (int t = 0; t < d / 2; ++t) fr[t] = (float)std::exp(-std::log(1e4) * t / (d / 2));
     std::vector<float> tf(d);
+    const float st = cfg.noise_scale * cfg.tau;
     for (int t = 0; t < d / 2; ++t) {
-      const double ang = (double)cfg.noise_scale * (double)cfg.tau * fr[t];
-      tf[t] = (float)std::cos(ang);
-      tf[d / 2 + t] = (float)std::sin(ang);
+      const float ang = st * fr[t];
+      tf[t] = std::cos(ang);
+      tf[d / 2 + t] = std::sin(ang);
     }
-    if ((r = dalloc(c, &c->noise_freq, fr.size() * 8)) || (r = fbuf(&c->tau_feat, tf.size()))) return bail(r);
+    if ((r = fbuf(&c->noise_freq, fr.size())) || (r = fbuf(&c->tau_feat, tf.size()))) return bail(r);
     if (cudaMemcpy(c->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(c->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(c->noise_freq, fr.data(), fr.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(c->noise_freq, fr.data(), fr.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(c->tau_feat, tf.data(), tf.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
       cuda_fail(c, cudaGetLastError(), "table upload");
       return bail(KF_E_CUDA);

@@ -491,7 +491,7 @@ void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* t
                          void* xb, float* ss, int* d_err, cudaStream_t s);
 void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, size_t total,
                        cudaStream_t s);
-void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, const float* tau_feat,
+void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, const float* tau_feat,
                        float scale, int d, void* feat, cudaStream_t s);
 void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
                     const float* g, float eps, void* out, cudaStream_t s);

@@ -148,17 +148,12 @@ void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, s
 // The angle (up to scale radians) is formed and reduced modulo 2 pi in fp64
 // (a few DFMAs), then sincosf runs on the reduced fp32 angle: the feature is
 // accurate to fp32 rounding without fp64 transcendentals.
-__device__ __forceinline__ void sincos_reduced(double ang, float* s, float* c) {
-  const double two_pi = 6.283185307179586;
-  const double k = rint(ang * (1.0 / two_pi));
-  const float r = (float)fma(-k, two_pi, ang);
-  sincosf(r, s, c);
-}
-
 // tau_feat: the temperature's encoding [cos | sin] of scale * tau * freq, the
-// same for every row (computed once per context)
+// same for every row (formed once per context).  The noise's angle is
+// (scale * z) * freq in fp32, in that order (the oracle's arithmetic), and
+// its cosine and sine come from sincosf (full argument reduction).
 template <typename TA>
-__global__ void k_noise_feat(int n, const float* __restrict__ noise, const double* __restrict__ freq,
+__global__ void k_noise_feat(int n, const float* __restrict__ noise, const float* __restrict__ freq,
                              const float* __restrict__ tau_feat, float scale, int d, TA* __restrict__ feat) {
   pdl_trigger();
   pdl_wait();
@@ -166,13 +161,14 @@ __global__ void k_noise_feat(int n, const float* __restrict__ noise, const doubl
   int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= n * half) return;
   int r = idx / half, t = idx - r * half;
+  const float ang = __fmul_rn(__fmul_rn(scale, noise[r]), freq[t]);
   float sz, cz;
-  sincos_reduced((double)scale * (double)noise[r] * freq[t], &sz, &cz);
+  sincosf(ang, &sz, &cz);
   feat[(size_t)r * d + t] = from_f<TA>(cz + tau_feat[t]);
   feat[(size_t)r * d + half + t] = from_f<TA>(sz + tau_feat[half + t]);
 }
 
-void launch_noise_feat(bool bf16, int n, const float* noise, const double* freq, const float* tau_feat,
+void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, const float* tau_feat,
                        float scale, int d, void* feat, cudaStream_t s) {
   if (n == 0) return;
   int tot = n * (d / 2);
