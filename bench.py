@@ -59,6 +59,8 @@ def parse():
     p.add_argument("--gemm", default="",
                    help="M,N,K[;M,N,K...]: the tcgen05 projection GEMM alone (kf_op_gemm_bf16), "
                         "automatic tiling against one CTA per tile")
+    p.add_argument("--flags", type=int, default=0,
+                   help="KF_FLAG_* bits for the decoders (e.g. 32: no skinny projections)")
     p.add_argument("--serving", action="store_true",
                    help="the G* teacher call and continuous batching (LM1B, batch 64)")
     return p.parse_args()
@@ -708,7 +710,8 @@ def main():
     stream = torch.cuda.Stream()
     max_b = max([B] + [e[1] for e in same])
     max_k = max([nout] + [max(e[2]) for e in same])
-    dec = kf.Decoder(model, weights, max_batch=max_b, max_k=max_k, stream=stream.cuda_stream)
+    dec = kf.Decoder(model, weights, max_batch=max_b, max_k=max_k, stream=stream.cuda_stream,
+                     flags=args.flags)
     dec.prefill(prompts)
 
     clk = Clocks(dev)
@@ -798,7 +801,7 @@ def main():
     for m, runs in by_model.items():
         wts = make_weights(m)
         d2 = kf.Decoder(m, wts, max_batch=max(r[1] for r in runs), max_k=max(max(r[2]) for r in runs),
-                        stream=stream.cuda_stream)
+                        stream=stream.cuda_stream, flags=args.flags)
         del wts
         for name, b, ks, wu, st in runs:
             configs[f"{name}_b{b}"] = measure_config(kf, d2, WORKLOADS[name], b, ks, pk, wu, st, stream)

@@ -54,6 +54,8 @@ extern "C" {
 #define KF_FLAG_NO_PDL 4         /* launch without programmatic dependent launch */
 #define KF_FLAG_NO_PERSISTENT_GEMM 16 /* bf16: one CTA per output tile even when the
                                     tiles exceed a wave (no persistent tile loop) */
+#define KF_FLAG_NO_SKINNY 32     /* bf16: keep the tcgen05 GEMMs for calls of at most
+                                    64 rows (no skinny warp-MMA projections)     */
 
 /*
  * Model and runtime configuration.  Table 4 gives the backbone (pre-norm

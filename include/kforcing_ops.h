@@ -17,12 +17,16 @@ extern "C" {
 #define KF_GEMM_SIMT 1      /* CUDA-core kernel, fp32 FMA in ascending k    */
 #define KF_GEMM_TCGEN05_PER_TILE 2 /* the tcgen05 kernel with one CTA per tile
                                       even past a wave of tiles            */
+#define KF_GEMM_SKINNY 3    /* M <= 64: warp-level MMA, 16 columns per CTA,
+                               K split over a cluster (the decode step at
+                               small batch)                                */
 
 /*
  * out[M][N] = A[M][K] . W[N][K]^T in fp32: the dense projections of the
  * backbone (Table 4: QKV, O, MLP) and the LM head are this contraction.
  * A, W: bf16, row-major, rows 16-byte aligned; K a multiple of 64 for
- * KF_GEMM_TCGEN05, N a multiple of 4.  out: fp32 row-major [M][N].  The first
+ * KF_GEMM_TCGEN05 and KF_GEMM_SKINNY (which also needs M <= 64), N a
+ * multiple of 4.  out: fp32 row-major [M][N].  The first
  * call on a device allocates a 4-byte device error word for that device that
  * lives until process exit; each call clears it on `stream` before its
  * kernel runs, and the kernel ORs its error bits into it (a bounded

@@ -84,6 +84,10 @@ struct kf_ctx {
   // workspaces
   int R_cap = 0, NR_cap = 0, prefill_rows = 0;
   bool fused = false;     // RMSNorm fused into the tcgen05 GEMMs (bf16, head_dim 64)
+  // The projections of the layers being enqueued run as skinny warp-MMA
+  // kernels (at most 64 rows, fused path): their norm consumers take the
+  // RMSNorm from their A rows, so no producer writes per-slot sums.
+  bool skinny = false;
   float* ss = nullptr;    // [rows][d/64] sums of squares of the residual stream
   float* x = nullptr;
   void *xn = nullptr, *qkv = nullptr, *attn = nullptr, *hmid = nullptr;
@@ -209,7 +213,11 @@ static void gemm(kf_ctx* c, int kind, int M, int N, int K, const void* A, int ld
   prof_begin(c, kind);
   bool use_tc = c->bf16 && !(c->cfg.flags & KF_FLAG_SIMT_GEMM) && tc_gemm_supported(g);
   g_gemm_flags = (c->cfg.flags & KF_FLAG_NO_PERSISTENT_GEMM) ? kGemmNoPersist : 0;
-  if (use_tc) {
+  if (c->skinny && e.kind != EPI_HEAD && e.kind != EPI_LOGITS) {
+    // every projection of a skinny enqueue must take this path: the fused
+    // RMSNorm's producers and consumers agree on it
+    if (!skinny_gemm_supported(g) || launch_gemm_skinny(g, c->d_err, c->stream) != 0) c->launch_failed = true;
+  } else if (use_tc) {
     if (launch_gemm_tc(g, c->d_err, c->stream) != 0) c->launch_failed = true;
   }
   else
@@ -262,7 +270,10 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   auto norm_in = [&](Epi& e) {
     e.ss_in = c->ss; e.nslot = d / 64; e.inv_d = 1.0f / d; e.eps = c->cfg.rms_eps;
   };
-  auto norm_out = [&](Epi& e) { e.xb_out = c->xn; e.ss_out = c->ss; e.nslot = d / 64; };
+  auto norm_out = [&](Epi& e) {
+    e.xb_out = c->xn; e.nslot = d / 64;
+    if (!c->skinny) e.ss_out = c->ss;
+  };
   // In one 128-row tile the projections stream their weights with few rows
   // to multiply them by: each prefetches the next projection's weights into
   // L2 (the last layer's MLP-down the first 32 MiB of the LM head).  Measured
@@ -289,6 +300,7 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
       eq.row_pos = c->row_pos; eq.page_table = c->d_page_table;
       eq.cos_t = c->cfg.pos_kind == KF_POS_ROPE ? c->rope_cos : nullptr; eq.sin_t = c->rope_sin;
       eq.d_err = c->d_err;
+      if (!groups) { eq.seq_len = c->d_len; eq.rows_per_seq = uniform_rows; }
       norm_in(eq);
       gemm(c, KF_KIND_GEMM_QKV, R, 3 * d, d, c->xn, d, w.wqkv, d, eq, pf ? w.wo : nullptr, (size_t)d * d * e2);
     } else {
@@ -342,6 +354,17 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   }
 }
 
+// Calls of at most 8 rows run their projections as skinny warp-MMA kernels
+// (weights staged before the dependency wait, no 128-row tcgen05 tiles).
+// Measured on the OWT-shaped model, microseconds per decode call, skinny vs
+// tcgen05: one sequence at k = 4 (8 rows) 366 vs 379; AR steps of 1 and 8
+// sequences 342 vs 349 and 373 vs 394; but 16 rows 411 vs 387, 32 rows 504
+// vs 400 and 64 rows 574 vs 441.
+constexpr int kSkinnyMaxRows = 8;
+static bool use_skinny(const kf_ctx* c, int R) {
+  return c->fused && R <= kSkinnyMaxRows && !(c->cfg.flags & KF_FLAG_NO_SKINNY);
+}
+
 // One decode step on the device: no host data dependence, so it can be
 // captured once per (B, P, k) and replayed.
 static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
@@ -353,6 +376,7 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   const bool mtp = c->mtp_k > 0 && k > 0;
   const int kz = mtp ? 1 : k;                      // noise rows per sequence
   const int S = P + kz, R = B * S, nout = k > 0 ? k : 1, nh = mtp ? B : B * nout;
+  c->skinny = use_skinny(c, R);
   prof_begin(c, KF_KIND_ROWMAP);
   launch_rowmap(B, P, kz, c->d_len, c->row_seq, c->row_pos, c->noise_map, c->head_map, s);
   prof_end(c);
@@ -376,7 +400,10 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
     Epi e2;
     e2.kind = EPI_NOISE_OUT; e2.x = c->x; e2.ldx = d; e2.bias = c->ne_b2;
     e2.row_map = c->noise_map; e2.row_pos = c->row_pos; e2.pos_emb = c->pos_emb;
-    if (c->fused) { e2.xb_out = c->xn; e2.ss_out = c->ss; e2.nslot = d / 64; }
+    if (c->fused) {
+      e2.xb_out = c->xn; e2.nslot = d / 64;
+      if (!c->skinny) e2.ss_out = c->ss;
+    }
     gemm(c, KF_KIND_NOISE_GEMM, B * kz, d, c->NH, c->nhid, c->NH, c->ne_w2, c->NH, e2,
          pf ? c->layers[0].wqkv : nullptr, (size_t)3 * d * d * c->esz);
   }
@@ -688,6 +715,7 @@ static int prefill_rows(kf_ctx* c, const std::vector<PrefillSeq>& seqs) {
                             c->stream));
     {
       PdlScope pdl(!(c->cfg.flags & KF_FLAG_NO_PDL));
+      c->skinny = use_skinny(c, R);
       launch_embed_tokens(c->bf16, R, c->row_tok, c->tok_emb, c->pos_emb, c->row_pos, c->V, c->d,
                           c->x, c->fused ? c->xn : nullptr, c->fused ? c->ss : nullptr, c->d_err,
                           c->stream);

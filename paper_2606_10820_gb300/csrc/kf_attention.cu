@@ -107,7 +107,6 @@ struct AttnSmem {
 
 template <typename TA, int HD, int R, int NBUF>
 __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
-  pdl_trigger();
   pdl_wait();
   using S = AttnSmem<TA, HD>;
   constexpr int KP = S::KP;
@@ -339,7 +338,6 @@ __global__ void __launch_bounds__(kAttnThreads) k_attention(AttnArgs a) {
 // merge the split partial softmaxes of one (row, head), splits in order
 template <typename TA>
 __global__ void k_attn_combine(AttnArgs a) {
-  pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x, h = blockIdx.y, dd = threadIdx.x;
   float M = -INFINITY;

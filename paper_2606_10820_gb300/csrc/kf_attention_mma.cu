@@ -115,7 +115,6 @@ __device__ __forceinline__ void merge_splits(const float* part_o, const float2* 
 template <int NBUF, bool TWO>
 __global__ void __launch_bounds__(kThr, NBUF == 1 ? (TWO ? 5 : 6) : 3)
 k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
-  pdl_trigger();
   extern __shared__ __align__(1024) uint8_t sm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
   __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(sm);   // [NBUF][128][64] swizzled

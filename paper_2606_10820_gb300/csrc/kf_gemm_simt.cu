@@ -10,7 +10,6 @@ namespace kf {
 
 template <typename TA>
 __global__ void __launch_bounds__(128) k_gemm_simt(GemmDesc g) {
-  pdl_trigger();
   pdl_wait();
   __shared__ float As[32][33];          // [row][k]
   __shared__ __align__(16) float Ws[32][132];  // [k][col]

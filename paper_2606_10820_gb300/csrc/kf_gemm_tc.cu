@@ -255,7 +255,6 @@ k_gemm_tc(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUt
   const int kb1 = min(kb_total, kb0 + g.kb_per_split);
   const int nkb = kb1 - kb0;                  // K atoms of this split
   const int nst = (nkb + AT - 1) / AT;        // pipeline stages (the last may be short)
-  pdl_trigger();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -576,7 +575,6 @@ k_gemm_tc_persist(const __grid_constant__ CUtensorMap map_a, const __grid_consta
   auto tile_m0 = [&](int t) { return (EPI == EPI_HEAD ? t % m_tiles : t / n_tiles) * kBM; };
   auto tile_n0 = [&](int t) { return (EPI == EPI_HEAD ? t / m_tiles : t % n_tiles) * BN; };
   const int nkb = g.K / kBK;
-  pdl_trigger();
   if (threadIdx.x == 0) {
     for (int i = 0; i < STAGES; ++i) {
       mbar_init(smem_u32(&full[i]), 1);
@@ -750,6 +748,12 @@ static bool make_map(CUtensorMap* m, const void* ptr, int rows, int cols, int ld
                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+// a K-major bf16 operand [rows][cols] (row pitch ld) read in boxes of 64
+// columns x box_rows rows, 128-byte swizzle (the skinny projections)
+bool encode_kmajor_bf16(CUtensorMap* m, const void* ptr, int rows, int cols, int ld, int box_rows) {
+  return get_encode() && make_map(m, ptr, rows, cols, ld, box_rows);
 }
 
 bool encode_rows_map_bf16(CUtensorMap* m, const void* base, uint64_t rows, int cols, int box_rows) {

@@ -162,6 +162,12 @@ struct Epi {
   const float* ss_in = nullptr;
   int nslot = 0;
   float inv_d = 0.f, eps = 0.f;
+  // EPI_QKV in a decode step (rows_per_seq rows per sequence, row r at
+  // position seq_len[r / rows_per_seq] + r % rows_per_seq): the skinny
+  // kernel reads positions and pages before its dependency wait (seq_len
+  // changes only at the step's commit), or NULL
+  const int32_t* seq_len = nullptr;
+  int rows_per_seq = 0;
 };
 
 // rsqrt(mean of squares + eps) of row `row` from its per-slot sums
@@ -381,17 +387,20 @@ __device__ __forceinline__ float4 add4(float4 a, float4 b) {
 }
 
 // ---------------------------------------------------------------- launches
-// Programmatic dependent launch: every kernel of the step lets its successor
-// launch as soon as all of its own CTAs are resident (pdl_trigger), and
-// waits for its predecessor grid to complete and publish its writes
-// (pdl_wait) before its first access to any buffer another kernel of the
-// step reads or writes.  Every kernel waits unconditionally, so completion
-// stays ordered along the chain.  Launched without the attribute both are
-// no-ops.
-__device__ __forceinline__ void pdl_trigger() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+// Programmatic dependent launch: every kernel of the step waits for its
+// predecessor grid to complete and publish its writes (pdl_wait) before its
+// first access to any buffer another kernel of the step reads or writes, and
+// only then lets its successor launch.  So one kernel at a time runs ahead:
+// the successor's CTAs become resident while this kernel works and load what
+// does not depend on it (weights, the cached K/V pages below the committed
+// length), then wait.  Triggering at kernel entry instead let four or five
+// kernels' CTAs pile up on the SMs and slowed the running kernel about 2x
+// (measured per phase with %globaltimer stamps at batch 1).  Every kernel
+// waits unconditionally, so completion stays ordered along the chain;
+// launched without the attribute both instructions are no-ops.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;\n\tgriddepcontrol.launch_dependents;" ::: "memory");
 }
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 extern thread_local bool g_pdl;   // launch with the programmatic-serialization attribute
 // tensor-core GEMM launch options for the launches made by this thread
@@ -434,6 +443,13 @@ void launch_gemm_simt(bool bf16, const GemmDesc& g, cudaStream_t s);
 // A rows readable up to round_up(M,128), W rows up to round_up(N,BN).
 bool tc_gemm_supported(const GemmDesc& g);
 int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s);
+
+// Skinny projections (kf_gemm_skinny.cu): M <= 64 rows on warp-level MMA,
+// weights staged before the dependency wait.  The fused RMSNorm scale comes
+// from the A rows themselves (epi.ss_in set means "normed input"; it is not
+// read), and residual producers must not ask for per-slot sums (ss_out NULL).
+bool skinny_gemm_supported(const GemmDesc& g);
+int launch_gemm_skinny(const GemmDesc& g, int* d_err, cudaStream_t s);
 
 struct AttnArgs {
   const float* q;          // [R][H][hd] (rotated, unscaled)

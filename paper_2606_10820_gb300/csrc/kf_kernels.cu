@@ -14,7 +14,10 @@ namespace kf {
 __global__ void k_rowmap(int B, int P, int k, const int32_t* __restrict__ len,
                          int32_t* row_seq, int32_t* row_pos, int32_t* noise_map,
                          int32_t* head_map) {
-  pdl_trigger();
+  // the step's later kernels launch only after this wait (pdl_wait triggers
+  // them): each may read the cached lengths before its own dependency wait
+  // (they change only at the step's commit, and the previous step's commit
+  // is complete once this wait returns)
   pdl_wait();
   int r = blockIdx.x * blockDim.x + threadIdx.x;
   int S = P + k;
@@ -79,7 +82,6 @@ __global__ void k_embed_pending(int P, int k, const int32_t* __restrict__ pendin
                                 const TA* __restrict__ emb, const float* __restrict__ pos_emb,
                                 const int32_t* __restrict__ row_pos, int V, int d, float* x,
                                 TA* xb, float* ss, int* d_err) {
-  pdl_trigger();
   pdl_wait();
   int b = blockIdx.x / P, i = blockIdx.x - b * P;
   int r = b * (P + k) + i;
@@ -90,7 +92,6 @@ template <typename TA>
 __global__ void k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
                                const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
                                int V, int d, float* x, TA* xb, float* ss, int* d_err) {
-  pdl_trigger();
   pdl_wait();
   int r = blockIdx.x;
   embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, xb, ss, d_err);
@@ -155,7 +156,6 @@ void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, s
 template <typename TA>
 __global__ void k_noise_feat(int n, const float* __restrict__ noise, const float* __restrict__ freq,
                              const float* __restrict__ tau_feat, float scale, int d, TA* __restrict__ feat) {
-  pdl_trigger();
   pdl_wait();
   int half = d / 2;
   int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -185,7 +185,6 @@ void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, 
 template <typename TA>
 __global__ void k_rmsnorm(const int32_t* __restrict__ row_map, const float* __restrict__ x, int d,
                           const float* __restrict__ g, float eps, TA* __restrict__ out) {
-  pdl_trigger();
   pdl_wait();
   int r = blockIdx.x;
   int src = row_map ? row_map[r] : r;
@@ -228,7 +227,6 @@ __global__ void k_rope_append(const TA* __restrict__ qkv, int d, int H,
                               const float* __restrict__ cos_t, const float* __restrict__ sin_t,
                               float* __restrict__ q, TA* __restrict__ kv, int layer, int n_pages,
                               const int32_t* __restrict__ page_table, int max_pages, int* d_err) {
-  pdl_trigger();
   pdl_wait();
   constexpr int HALF = HD / 2;
   int r = blockIdx.x;
@@ -330,7 +328,6 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
               const TA* __restrict__ w_head_all, int V, float inv_tau, int map_kind,
               const float* __restrict__ noise, int32_t* __restrict__ tokens, int mtp_rows,
               size_t head_stride, const int* __restrict__ err) {
-  pdl_trigger();
   pdl_wait();
   // one block per mapped row; MTP (mtp_rows = B > 0): block j B + b is head j
   // of sequence b (records in that order), hidden row b, weights w_head + j
@@ -564,7 +561,6 @@ void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, c
 // become the next step's pending tokens (App. C.1 fixed stride).
 __global__ void k_commit(int B, int P, int nout, const int32_t* __restrict__ tokens,
                          int32_t* pending, int pend_stride, int32_t* len) {
-  pdl_trigger();
   pdl_wait();
   int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
@@ -585,7 +581,6 @@ namespace kf {
 // fp32 -> storage type (round to nearest even for bf16)
 template <typename T>
 __global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, size_t n) {
-  pdl_trigger();
   pdl_wait();
   size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   size_t stride = (size_t)gridDim.x * blockDim.x;

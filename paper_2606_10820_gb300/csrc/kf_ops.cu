@@ -105,6 +105,11 @@ extern "C" int kf_op_gemm_bf16(int32_t impl, int32_t M, int32_t N, int32_t K, co
     // each call starts with a clear error word (kf_op_status reads it)
     if (cudaMemsetAsync(err, 0, sizeof(int), s) != cudaSuccess) return KF_E_CUDA;
     if (launch_gemm_tc(g, err, s) != 0) return KF_E_CUDA;
+  } else if (impl == KF_GEMM_SKINNY) {
+    if (!skinny_gemm_supported(g)) return KF_E_ARG;
+    int* err = op_error_word(s);
+    if (!err) return KF_E_CUDA;
+    if (launch_gemm_skinny(g, err, s) != 0) return KF_E_CUDA;
   } else if (impl == KF_GEMM_SIMT) {
     launch_gemm_simt(true, g, s);
   } else {

@@ -85,7 +85,6 @@ constexpr size_t smem_bytes() { return (size_t)kRows * kHD * 2 + 2 * 2 * (size_t
 }  // namespace
 
 __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
-  pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(128) uint8_t sm[];
   __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(sm);       // [64][64] swizzled
@@ -335,7 +334,6 @@ constexpr size_t tc_smem_bytes() {
 __global__ void __launch_bounds__(kTcThreads, 1)
 k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                      const __grid_constant__ CUtensorMap map_v, TrainAttnArgs a, int* d_err) {
-  pdl_trigger();
   extern __shared__ __align__(1024) uint8_t tsm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tsm_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(sm);

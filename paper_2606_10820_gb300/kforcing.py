@@ -23,6 +23,7 @@ KF_POS_ROPE, KF_POS_LEARNED = 0, 1
 KF_DTYPE_FP32, KF_DTYPE_BF16 = 0, 1
 KF_MAP_ICDF, KF_MAP_ARGMAX = 0, 1
 KF_FLAG_NO_GRAPH, KF_FLAG_SIMT_GEMM, KF_FLAG_NO_PDL, KF_FLAG_NO_PERSISTENT_GEMM = 1, 2, 4, 16
+KF_FLAG_NO_SKINNY = 32
 KIND_NAMES = ["rowmap", "embed", "noise_gemm", "rmsnorm", "gemm_qkv", "rope_kv", "attention",
               "attn_combine", "gemm_o", "gemm_up", "gemm_down", "head_norm", "gemm_head",
               "head_select", "commit"]

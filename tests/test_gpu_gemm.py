@@ -28,6 +28,20 @@ SHAPES = [
 
 PERSISTENT = [(2100, 2340, 768), (4096, 2304, 768), (4096, 3072, 768)]
 
+# the skinny warp-MMA kernel (M <= 64): one K range per CTA, or K split over
+# clusters of 2, 4 and 8 CTAs; ragged M (one 8-row box, several n-blocks)
+# and N (the last 16-column block partly past N)
+SKINNY = [
+    (1, 128, 64),        # one row, one K atom
+    (8, 2304, 768),      # OWT batch 1, k = 4 QKV rows
+    (6, 3072, 768),      # MLP-up, a partial 8-row box
+    (64, 768, 3072),     # batch 8, k = 4 MLP-down: K over a cluster of 8
+    (33, 768, 768),      # five n-blocks, K split 2
+    (17, 200, 128),      # N not a multiple of 16
+    (40, 768, 832),      # 13 K atoms: no power-of-two split divides them
+    (16, 1000, 3072),    # K split 4, ragged N
+]
+
 
 @pytest.fixture(scope="module")
 def env():
@@ -88,3 +102,19 @@ def test_gemm_repeat_is_deterministic(env):
     a = _run(torch, lib, 0, A, W)
     b = _run(torch, lib, 0, A, W)
     assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("M,N,K", SKINNY)
+def test_skinny_gemm_matches_fp32_matmul(env, M, N, K):
+    torch, lib = env
+    g = torch.Generator(device="cuda").manual_seed(M * 11 + N * 5 + K)
+    A = (torch.randn(M, K, device="cuda", generator=g) * 0.5).to(torch.bfloat16)
+    W = (torch.randn(N, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    ref = (A.double() @ W.double().T).float()
+    scale = ref.abs().max().item()
+    out = _run(torch, lib, 3, A, W)
+    assert torch.isfinite(out).all()
+    err = (out - ref).abs().max().item()
+    assert err <= 1e-4 * scale + 1e-6, (err, scale)
+    # split partials are summed in split order: identical bits each run
+    assert torch.equal(out, _run(torch, lib, 3, A, W))

@@ -523,3 +523,33 @@ def test_persistent_gemm_equals_per_tile_model(kf):
     pick = [0, 131, 511]
     worst, slots, mism, bad = _sampled(kf, cfg, w, prompts, pick, [4, 4, 0], 4, 23)
     assert worst <= LOGIT_TOL and bad == 0
+
+
+def test_skinny_and_tcgen05_small_batch(kf, lm1b_weights):
+    """Calls of at most 64 rows run their projections as skinny warp-MMA
+    kernels; KF_FLAG_NO_SKINNY keeps the tcgen05 GEMMs.  Batch 8 reaches
+    exactly 64 rows at k = 4 (P = 4 pending + 4 noise rows per sequence).
+    Both paths stay within tolerance of the oracle, and of each other."""
+    cfg = LM1B
+    prompts = make_prompts([32, 5, 17, 32, 40, 9, 23, 32], cfg.vocab)
+    logits = []
+    for flags in (0, kf.KF_FLAG_NO_SKINNY):
+        dec, recs = _run(kf, cfg, lm1b_weights, prompts, [4, 4, 0, 4, 2], max_k=4, seed=31, flags=flags)
+        worst, slots, mism, bad = _bf16_check(recs)
+        assert worst <= LOGIT_TOL and bad == 0, (flags, worst, bad)
+        logits.append(recs[0][4])
+        dec.close()
+    rng = logits[1].max(axis=-1, keepdims=True) - logits[1].min(axis=-1, keepdims=True)
+    assert (np.abs(logits[0] - logits[1]) / rng).max() <= LOGIT_TOL
+
+
+def test_owt_batch1_skinny_rows(kf):
+    """One sequence of the OWT-shaped model: 8, 6 and 2 rows per call (k = 4,
+    k = 2 and the AR step after a k = 2 step), all under one 8-row A box."""
+    cfg = OWT.replace(n_layer=2)
+    w = make_weights(cfg)
+    prompts = make_prompts([300], cfg.vocab)
+    dec, recs = _run(kf, cfg, w, prompts, [4, 4, 2, 0, 4], max_k=4, seed=33)
+    worst, slots, mism, bad = _bf16_check(recs)
+    assert worst <= LOGIT_TOL and bad == 0
+    dec.close()
