@@ -354,13 +354,13 @@ static void enqueue_layers(kf_ctx* c, int R, int n_groups, const int4* groups, i
   }
 }
 
-// Calls of at most 8 rows run their projections as skinny warp-MMA kernels
+// Calls of at most 16 rows run their projections as skinny warp-MMA kernels
 // (weights staged before the dependency wait, no 128-row tcgen05 tiles).
 // Measured on the OWT-shaped model, microseconds per decode call, skinny vs
-// tcgen05: one sequence at k = 4 (8 rows) 366 vs 379; AR steps of 1 and 8
-// sequences 342 vs 349 and 373 vs 394; but 16 rows 411 vs 387, 32 rows 504
-// vs 400 and 64 rows 574 vs 441.
-constexpr int kSkinnyMaxRows = 8;
+// tcgen05 (same box): 2 sequences at k = 4 (16 rows) 374.7 vs 388.3, AR step
+// of 16 sequences 382.4 vs 396.3; but 32 rows 470.7 vs 401.0 and 64 rows
+// 564.0 vs 442.8 (a 16-column CTA re-reads the A rows once per 16 columns).
+constexpr int kSkinnyMaxRows = 16;
 static bool use_skinny(const kf_ctx* c, int R) {
   return c->fused && R <= kSkinnyMaxRows && !(c->cfg.flags & KF_FLAG_NO_SKINNY);
 }

@@ -424,7 +424,15 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
         acc[4] += u1.x * wt[w]; acc[5] += u1.y * wt[w]; acc[6] += u1.z * wt[w]; acc[7] += u1.w * wt[w];
       }
       const int row = row0 + r;
-      if (a.n_split == 1) {
+      if (a.cluster_merge) {
+        // this split's partial (base-2 units) for the cluster merge below;
+        // past the 4-warp merge's buffers (Ow and ML end 16.5 KB in)
+        float* Ps = reinterpret_cast<float*>(sm + 17408);          // [16][64]
+        float2* MLs = reinterpret_cast<float2*>(Ps + kQRows * kHD);  // [16]
+        *reinterpret_cast<float4*>(Ps + r * kHD + d0) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+        *reinterpret_cast<float4*>(Ps + r * kHD + d0 + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+        if (d0 == 0) MLs[r] = make_float2(M, L);
+      } else if (a.n_split == 1) {
         const float inv = 1.f / L;
         uint4 pk;
         pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
@@ -442,6 +450,46 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
         if (d0 == 0) a.part_ml[((size_t)split * a.R + row) * a.H + h] = make_float2(M * 0.6931471805599453f, L);
       }
     }
+  }
+  if (a.cluster_merge) {
+    // The key splits of this (group, head) are one cluster (rank = split):
+    // after the barrier CTA q merges rows q, q + n_split, ... reading every
+    // split's partial from its shared memory in split order; the second
+    // barrier keeps each CTA's partial alive until all have read it.
+    cluster_sync();
+    const int r = t >> 3, d0 = (t & 7) * 8;
+    if (r < nr && r % a.n_split == split) {
+      const float* Ps = reinterpret_cast<const float*>(sm + 17408);
+      const float2* MLs = reinterpret_cast<const float2*>(Ps + kQRows * kHD);
+      float M = -INFINITY, L = 0.f, acc[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+      for (int sp = 0; sp < a.n_split; ++sp) {
+        const float2 ml = ld_dsmem2(smem_u32(MLs + r), (uint32_t)sp);
+        if (ml.x == -INFINITY) continue;            // no visible key in this split
+        const float4 u0 = ld_dsmem4(smem_u32(Ps + r * kHD + d0), (uint32_t)sp);
+        const float4 u1 = ld_dsmem4(smem_u32(Ps + r * kHD + d0 + 4), (uint32_t)sp);
+        const float Mn = fmaxf(M, ml.x);
+        const float cs = (M == -INFINITY) ? 0.f : ex2(M - Mn);
+        const float w = ex2(ml.x - Mn);
+        M = Mn;
+        L = L * cs + ml.y * w;
+        acc[0] = acc[0] * cs + u0.x * w; acc[1] = acc[1] * cs + u0.y * w;
+        acc[2] = acc[2] * cs + u0.z * w; acc[3] = acc[3] * cs + u0.w * w;
+        acc[4] = acc[4] * cs + u1.x * w; acc[5] = acc[5] * cs + u1.y * w;
+        acc[6] = acc[6] * cs + u1.z * w; acc[7] = acc[7] * cs + u1.w * w;
+      }
+      const float inv = 1.f / L;
+      uint4 pk;
+      pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+      pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+      pk.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+      pk.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+      *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) + (size_t)(row0 + r) * a.H * kHD +
+                                h * kHD + d0) = pk;
+    }
+    cluster_sync();
+    return;
   }
   if constexpr (NBUF > 1) {
     // the last split CTA of this (group, head) to finish merges the
@@ -464,11 +512,29 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
 }
 
 template <int NBUF, bool TWO>
-static void launch_nb(const CUtensorMap& map, const AttnArgs& a, int n_groups, cudaStream_t s) {
+static int launch_nb(const CUtensorMap& map, const AttnArgs& a, int n_groups, cudaStream_t s) {
   static PerDevice attr;
   const size_t smem = smem_bytes(NBUF, a.pg_cap);
   set_smem_attr(attr, k_attention_mma<NBUF, TWO>, smem);
-  kf_launch(k_attention_mma<NBUF, TWO>, dim3(n_groups, a.H, a.n_split), dim3(kThr), smem, s, map, a);
+  if (!a.cluster_merge) {
+    kf_launch(k_attention_mma<NBUF, TWO>, dim3(n_groups, a.H, a.n_split), dim3(kThr), smem, s, map, a);
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_groups, a.H, a.n_split);
+  cfg.blockDim = dim3(kThr);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 1;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = a.n_split;
+  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = g_pdl ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, k_attention_mma<NBUF, TWO>, map, a) == cudaSuccess ? 0 : -1;
 }
 
 bool attention_mma_supported(bool bf16, int hd, int rows) { return bf16 && hd == kHD && rows <= kQRows; }
@@ -489,10 +555,12 @@ int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_key
   // 256 481k -> 493k tokens/s; batch 32 (384 CTAs) 239k with two buffers,
   // 209k with one
   const bool one = keys <= kTile || ctas > 3L * num_sms;
-  // CTAs with two buffers merge their own splits; single-buffer CTAs (80
-  // registers) leave it to k_attn_combine
-  if (one || a.n_split == 1) a.split_count = nullptr;
-  *merged = a.split_count != nullptr;
+  // the key splits of each (group, head) run as one cluster (at most 4
+  // CTAs) and merge in the kernel
+  a.split_count = nullptr;
+  a.cluster_merge = a.n_split > 1 && a.n_split <= 8 ? 1 : 0;
+  if (a.n_split > 8) return -1;
+  *merged = a.cluster_merge != 0;
   a.pg_cap = one ? 0 : ceil_div(keys, kPage);   // staged page ids (two-buffer CTAs)
   // this layer's K/V pages as rows of 64 bf16: ((page * 2 + kv) * H + head) * 16 + key
   const size_t layer_elems = (size_t)a.n_pages * 2 * a.H * kPage * kHD;
@@ -500,14 +568,8 @@ int launch_attention_mma(const AttnArgs& a0, int n_groups, int rows, int max_key
   if (!encode_rows_map_bf16(&map, static_cast<const __nv_bfloat16*>(a.kv) + (size_t)a.layer * layer_elems,
                             (uint64_t)a.n_pages * 2 * a.H * kPage, kHD, kPage))
     return -1;
-  if (one) {
-    if (two) launch_nb<1, true>(map, a, n_groups, s);
-    else launch_nb<1, false>(map, a, n_groups, s);
-  } else {
-    if (two) launch_nb<2, true>(map, a, n_groups, s);
-    else launch_nb<2, false>(map, a, n_groups, s);
-  }
-  return 0;
+  if (one) return two ? launch_nb<1, true>(map, a, n_groups, s) : launch_nb<1, false>(map, a, n_groups, s);
+  return two ? launch_nb<2, true>(map, a, n_groups, s) : launch_nb<2, false>(map, a, n_groups, s);
 }
 
 }  // namespace kf

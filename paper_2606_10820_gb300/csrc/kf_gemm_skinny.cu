@@ -321,6 +321,25 @@ k_gemm_skinny(const __grid_constant__ CUtensorMap map_a, const __grid_constant__
   }
   __syncthreads();
 
+  // this thread's outputs summed over the splits (QKV: both members of a
+  // RoPE pair), then the peers may leave once every CTA has read (the
+  // cluster barrier's arrive here, its wait after the stores)
+  float va[kSkMaxE], vb[kSkMaxE];
+#pragma unroll
+  for (int j = 0; j < kSkMaxE; ++j) {
+    const int i = tid + j * kSkThreads;
+    va[j] = vb[j] = 0.f;
+    if (!ok || i >= ne) continue;
+    const int m = split + (i / per_row) * S;
+    if (EPI == EPI_QKV) {
+      va[j] = split_sum(P, m * 16 + (i & 7), S);
+      vb[j] = split_sum(P, m * 16 + (i & 7) + 8, S);
+    } else if (w0 + (i & 15) < g.N) {
+      va[j] = split_sum(P, m * 16 + (i & 15), S);
+    }
+  }
+  if (S > 1) cluster_arrive();
+
   if (ok) {
 #pragma unroll
     for (int j = 0; j < kSkMaxE; ++j) {
@@ -329,7 +348,7 @@ k_gemm_skinny(const __grid_constant__ CUtensorMap map_a, const __grid_constant__
       const int m = split + (i / per_row) * S;
       if (EPI == EPI_QKV) {
         const int pi = i & 7;
-        float a = split_sum(P, m * 16 + pi, S), b = split_sum(P, m * 16 + pi + 8, S);
+        float a = va[j], b = vb[j];
         if (g.norm) { a *= rinv[m]; b *= rinv[m]; }
         const int gc = j0 + pi;
         const int col = hb * 64 + gc;
@@ -354,7 +373,7 @@ k_gemm_skinny(const __grid_constant__ CUtensorMap map_a, const __grid_constant__
         const int c = i & 15;
         const int n = w0 + c;
         if (n >= g.N) continue;
-        float v = split_sum(P, m * 16 + c, S);
+        float v = va[j];
         if (EPI == EPI_STORE_F32) {
           e.outf[(size_t)m * e.ldo + n] = v;
         } else if (EPI == EPI_STORE) {
@@ -377,7 +396,7 @@ k_gemm_skinny(const __grid_constant__ CUtensorMap map_a, const __grid_constant__
     }
   }
   // no CTA leaves while a peer may still read its partial
-  if (S > 1) cluster_sync();
+  if (S > 1) cluster_wait();
 }
 
 // ------------------------------------------------------------ host side

@@ -473,6 +473,9 @@ struct AttnArgs {
   int pg_cap = 0;                // pages of one CTA's key range (set by the launcher)
   int* split_count = nullptr;    // [groups][H] zeroed counters: the warp-MMA kernel merges
                                  // its own splits (no k_attn_combine launch)
+  int cluster_merge = 0;           // warp-MMA kernel, n_split > 1: the key splits of a
+                                   // (group, head) form a thread-block cluster and merge
+                                   // their partial softmaxes over distributed shared memory
   const int32_t* order = nullptr;  // uniform groups: group g is sequence order[g] (a
                                    // permutation, longest first: each head's longest CTAs
                                    // start first and the grid's last wave holds the
