@@ -44,57 +44,81 @@ void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, 
 // x[r] = E[tok] (+ pos_emb[pos]).  With the fused RMSNorm (xb != NULL) the
 // row is also written as bf16 into xb and the sum of squares of each of its
 // 64-column slots into ss[r][d/64] (warp partials over 32 columns, then the
-// pair of a slot added in order).
+// pair of a slot added in order).  The token id and its embedding row do not
+// depend on the step's earlier kernels: a thread loads its (at most
+// kEmbedPer) columns before the dependency wait, all loads in flight at once.
+constexpr int kEmbedThreads = 128;
+constexpr int kEmbedPer = 8;           // d <= 1024 kept in registers
+
 template <typename TA>
-__device__ void embed_row(int r, int tok, int pos, const TA* __restrict__ emb,
+__device__ void embed_row(int r, int tok, const int32_t* __restrict__ row_pos, const TA* __restrict__ emb,
                           const float* __restrict__ pos_emb, int V, int d, float* x, TA* xb,
                           float* ss, int* d_err) {
   __shared__ float part[128];          // d <= 4096
-  float* o = x + (size_t)r * d;
   const bool good = tok >= 0 && tok < V;
-  if (!good && threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
   const TA* e = emb + (size_t)(good ? tok : 0) * d;
-  const float* p = pos_emb ? pos_emb + (size_t)pos * d : nullptr;
   const int lane = threadIdx.x & 31;
-  for (int c0 = threadIdx.x - lane; c0 < d; c0 += blockDim.x) {
+  const bool held = d <= kEmbedPer * kEmbedThreads;
+  float v[kEmbedPer];
+#pragma unroll
+  for (int j = 0; j < kEmbedPer; ++j) {
+    const int c = threadIdx.x + j * kEmbedThreads;
+    v[j] = held && good && c < d ? to_f(e[c]) : 0.f;
+  }
+  pdl_wait();
+  if (!good && threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
+  float* o = x + (size_t)r * d;
+  const float* p = pos_emb ? pos_emb + (size_t)row_pos[r] * d : nullptr;
+  for (int c0 = threadIdx.x - lane, j = 0; c0 < d; c0 += kEmbedThreads, ++j) {
     const int c = c0 + lane;
-    float v = 0.f;
+    float w = 0.f;
     if (c < d) {
-      v = good ? to_f(e[c]) + (p ? p[c] : 0.f) : 0.f;
-      o[c] = v;
-      if (xb) xb[(size_t)r * d + c] = from_f<TA>(v);
+      float base = 0.f;
+      if (held) {
+#pragma unroll
+        for (int q = 0; q < kEmbedPer; ++q)
+          if (q == j) base = v[q];
+      } else {
+        base = good ? to_f(e[c]) : 0.f;
+      }
+      w = good ? base + (p ? p[c] : 0.f) : 0.f;
+      o[c] = w;
+      if (xb) xb[(size_t)r * d + c] = from_f<TA>(w);
     }
     if (ss) {
-      float q = v * v;
+      float q = w * w;
       for (int k = 16; k > 0; k >>= 1) q += __shfl_xor_sync(0xffffffffu, q, k);
       if (lane == 0) part[c0 / 32] = q;
     }
   }
   if (ss) {
     __syncthreads();
-    for (int sl = threadIdx.x; sl < d / 64; sl += blockDim.x)
+    for (int sl = threadIdx.x; sl < d / 64; sl += kEmbedThreads)
       ss[(size_t)r * (d / 64) + sl] = part[2 * sl] + part[2 * sl + 1];
   }
 }
 
+// the pending ids were written by the previous step's commit, which has
+// completed before any kernel after the step's first one launches
 template <typename TA>
-__global__ void k_embed_pending(int P, int k, const int32_t* __restrict__ pending, int pend_stride,
-                                const TA* __restrict__ emb, const float* __restrict__ pos_emb,
-                                const int32_t* __restrict__ row_pos, int V, int d, float* x,
-                                TA* xb, float* ss, int* d_err) {
-  pdl_wait();
+__global__ void __launch_bounds__(kEmbedThreads)
+k_embed_pending(int P, int k, const int32_t* __restrict__ pending, int pend_stride,
+                const TA* __restrict__ emb, const float* __restrict__ pos_emb,
+                const int32_t* __restrict__ row_pos, int V, int d, float* x,
+                TA* xb, float* ss, int* d_err) {
   int b = blockIdx.x / P, i = blockIdx.x - b * P;
   int r = b * (P + k) + i;
-  embed_row<TA>(r, pending[b * pend_stride + i], row_pos[r], emb, pos_emb, V, d, x, xb, ss, d_err);
+  embed_row<TA>(r, pending[b * pend_stride + i], row_pos, emb, pos_emb, V, d, x, xb, ss, d_err);
 }
 
+// the row tokens are copied from the host before the launch
 template <typename TA>
-__global__ void k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
-                               const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
-                               int V, int d, float* x, TA* xb, float* ss, int* d_err) {
-  pdl_wait();
+__global__ void __launch_bounds__(kEmbedThreads)
+k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
+               const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
+               int V, int d, float* x, TA* xb, float* ss, int* d_err) {
   int r = blockIdx.x;
-  embed_row<TA>(r, row_tok[r], row_pos[r], emb, pos_emb, V, d, x, xb, ss, d_err);
+  embed_row<TA>(r, row_tok[r], row_pos, emb, pos_emb, V, d, x, xb, ss, d_err);
 }
 
 void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
@@ -102,11 +126,11 @@ void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending
                           int V, int d, float* x, void* xb, float* ss, int* d_err, cudaStream_t s) {
   if (B * P == 0) return;
   if (bf16)
-    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(128), 0, s, P, k, pending,
+    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(kEmbedThreads), 0, s, P, k, pending,
               pend_stride, (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x,
               (__nv_bfloat16*)xb, ss, d_err);
   else
-    kf_launch(k_embed_pending<float>, dim3(B * P), dim3(128), 0, s, P, k, pending, pend_stride,
+    kf_launch(k_embed_pending<float>, dim3(B * P), dim3(kEmbedThreads), 0, s, P, k, pending, pend_stride,
               (const float*)tok_emb, pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
 }
 
@@ -115,11 +139,11 @@ void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* t
                          void* xb, float* ss, int* d_err, cudaStream_t s) {
   if (R == 0) return;
   if (bf16)
-    kf_launch(k_embed_tokens<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_tok,
+    kf_launch(k_embed_tokens<__nv_bfloat16>, dim3(R), dim3(kEmbedThreads), 0, s, row_tok,
               (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x, (__nv_bfloat16*)xb, ss,
               d_err);
   else
-    kf_launch(k_embed_tokens<float>, dim3(R), dim3(128), 0, s, row_tok, (const float*)tok_emb,
+    kf_launch(k_embed_tokens<float>, dim3(R), dim3(kEmbedThreads), 0, s, row_tok, (const float*)tok_emb,
               pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
 }
 
@@ -182,37 +206,65 @@ void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, 
 
 // --------------------------------------------------------------- RMSNorm
 // out[r] = x[src] / sqrt(mean(x[src]^2) + eps) * g   (Table 4 pre-norm)
+constexpr int kNormThreads = 128;
+constexpr int kNormPer = 8;            // d <= 1024 kept in registers
 template <typename TA>
-__global__ void k_rmsnorm(const int32_t* __restrict__ row_map, const float* __restrict__ x, int d,
-                          const float* __restrict__ g, float eps, TA* __restrict__ out) {
+__global__ void __launch_bounds__(kNormThreads)
+k_rmsnorm(const int32_t* __restrict__ row_map, const float* __restrict__ x, int d,
+          const float* __restrict__ g, float eps, TA* __restrict__ out) {
+  const bool held = d <= kNormPer * kNormThreads;
+  float gv[kNormPer], xv[kNormPer];
+#pragma unroll
+  for (int j = 0; j < kNormPer; ++j) {     // the gains before the dependency
+    const int c = threadIdx.x + j * kNormThreads;
+    gv[j] = held && c < d ? g[c] : 0.f;
+  }
   pdl_wait();
   int r = blockIdx.x;
   int src = row_map ? row_map[r] : r;
   const float* xr = x + (size_t)src * d;
   float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += xr[c] * xr[c];
+  if (held) {
+#pragma unroll
+    for (int j = 0; j < kNormPer; ++j) {
+      const int c = threadIdx.x + j * kNormThreads;
+      xv[j] = c < d ? xr[c] : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < kNormPer; ++j) ss += xv[j] * xv[j];
+  } else {
+    for (int c = threadIdx.x; c < d; c += kNormThreads) ss += xr[c] * xr[c];
+  }
   __shared__ float red[32];
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
   if (threadIdx.x < 32) {
-    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    float v = threadIdx.x < (kNormThreads >> 5) ? red[threadIdx.x] : 0.f;
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     if (threadIdx.x == 0) red[0] = v;
   }
   __syncthreads();
   float inv = rsqrtf(red[0] / (float)d + eps);
   TA* o = out + (size_t)r * d;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = from_f<TA>(xr[c] * inv * g[c]);
+  if (held) {
+#pragma unroll
+    for (int j = 0; j < kNormPer; ++j) {
+      const int c = threadIdx.x + j * kNormThreads;
+      if (c < d) o[c] = from_f<TA>(xv[j] * inv * gv[j]);
+    }
+  } else {
+    for (int c = threadIdx.x; c < d; c += kNormThreads) o[c] = from_f<TA>(xr[c] * inv * g[c]);
+  }
 }
 
 void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
                     const float* g, float eps, void* out, cudaStream_t s) {
   if (R == 0) return;
   if (bf16)
-    kf_launch(k_rmsnorm<__nv_bfloat16>, dim3(R), dim3(128), 0, s, row_map, x, d, g, eps, (__nv_bfloat16*)out);
+    kf_launch(k_rmsnorm<__nv_bfloat16>, dim3(R), dim3(kNormThreads), 0, s, row_map, x, d, g, eps, (__nv_bfloat16*)out);
   else
-    kf_launch(k_rmsnorm<float>, dim3(R), dim3(128), 0, s, row_map, x, d, g, eps, (float*)out);
+    kf_launch(k_rmsnorm<float>, dim3(R), dim3(kNormThreads), 0, s, row_map, x, d, g, eps, (float*)out);
 }
 
 // ------------------------------------------------------ RoPE + KV append
