@@ -217,8 +217,10 @@ k_attention_mma(const __grid_constant__ CUtensorMap map_kv, AttnArgs a) {
     if (go) {
       const int row = (page * 2 * a.H + h) * kPage;   // K rows; V rows follow H pages later
       const uint32_t off = (uint32_t)(buf * kTileBytes + lane * kPageBytes);
-      tma_load_2d(smem_u32(Ks) + off, &map_kv, bar, 0, row);
-      tma_load_2d(smem_u32(Vs) + off, &map_kv, bar, 0, row + a.H * kPage);
+      // each K/V byte is read once per step: evict first
+      const uint64_t pol = l2_evict_first_policy();
+      tma_load_2d_hint(smem_u32(Ks) + off, &map_kv, bar, 0, row, pol);
+      tma_load_2d_hint(smem_u32(Vs) + off, &map_kv, bar, 0, row + a.H * kPage, pol);
     }
     if constexpr (NBUF == 1) {
       // the next tile's page ids, consumed at its issue after this tile's compute
