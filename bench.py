@@ -732,6 +732,21 @@ def main():
               "calls_per_step": ar_calls,
               "step_roofline_frac": generation_roofline_s(model, prompts, 0, ar_calls, pk) * 1e3 / ar_ms}
 
+    # prefill of the workload's prompts (kf_prefill from host prompt ids: page
+    # allocation, the copies and the chunked forward over every prompt token
+    # but each sequence's last), wall clock; not part of the decode metric
+    pre_tok = sum(len(p) - 1 for p in prompts)
+    for _ in range(2):
+        dec.prefill(prompts)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(3):
+        dec.prefill(prompts)
+    torch.cuda.synchronize()
+    pre_ms = (time.perf_counter() - t0) * 1000.0 / 3
+    prefill = {"value": pre_tok / (pre_ms / 1e3), "unit": "prompt tokens/s", "tokens": pre_tok,
+               "ms": pre_ms, "timing": "wall clock around kf_prefill, host prompt ids in"}
+
     # per-kernel times of one call in the middle of the generation
     # (kf_profile_step: the call replayed as a graph whose event-record nodes
     # bracket each launch, without programmatic dependent launch); launches
@@ -829,6 +844,7 @@ def main():
             "clocks": clocks,
             "gpu_launches": launches_per_step * args.steps,
             "kernel_ms_mid_call": {kn: round(v, 4) for kn, v in tot_ms.items() if v > 0},
+            "prefill": prefill,
             "configs": configs,
         }
         print(json.dumps(line))
