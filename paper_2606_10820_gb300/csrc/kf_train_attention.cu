@@ -296,16 +296,19 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
 //               (128-byte swizzle) into a four-stage ring;
 //   warp 1      one thread issues tcgen05.mma: S_j = Q K_j^T (M = 128 rows,
 //               N = 128 keys, K = 64) into one of two TMEM buffers, and
-//               O_j = P_j V_j (M = 128, N = 64, K = 128 keys; V is the
-//               MN-major operand as loaded) into one of two more;
+//               O += P_j V_j (M = 128, N = 64, K = 128 keys; V is the
+//               MN-major operand as loaded) into one TMEM accumulator;
 //   warps 2..9  two threads per query row (TMEM lane), each with half of
 //               its keys and of its output (four threads measured 5 % slower:
 //               the per-tile chain of waits and barriers, not the arithmetic,
 //               bounds the softmax): mask S_j, share the row max
-//               through shared memory, keep the running max m and their part
-//               of the sum l, write P_j = exp2(S_j - m) as bf16 into shared
-//               memory (K-major, swizzled: the A operand of P V) and fold
-//               O_j into their fp32 output dims, o <- o exp2(m_prev - m) + O_j.
+//               through shared memory, keep a reference max m and their
+//               part of the sum l, and write P_j = exp2(S_j - m) as bf16 into
+//               shared memory (K-major, swizzled: the A operand of P V).  m
+//               is raised only when a tile's max exceeds it by more than 2^8
+//               (P stays below 256); then O in TMEM and l are scaled to the
+//               new m before P_j is released.  At the end O / l is the row's
+//               output.
 // S of tile j + 1 is computed while the softmax works on tile j.  Every
 // wait is bounded; a wait that runs out sets the error word and ends the
 // CTA's loops.
@@ -349,8 +352,7 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
   uint64_t* s_full = kv_empty + kTcStages;           // [2]
   uint64_t* p_full = s_full + 2;                     // [2]: P_j written (and S_j read)
   uint64_t* o_full = p_full + 2;                     // [2]
-  uint64_t* o_empty = o_full + 2;                    // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_empty + 2);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 2);
   int* s_rng = reinterpret_cast<int*>(tmem_slot + 1);   // cmax, w1lo, w1hi, w2lo, w2hi, cmin
   int* s_cnt = s_rng + 6;                                // tiles whose K/V the MMA has taken
   volatile int* s_abort = s_cnt + 1;                     // a softmax thread's wait ran out
@@ -375,7 +377,6 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       mbar_init(smem_u32(&s_full[i]), 1);
       mbar_init(smem_u32(&p_full[i]), 1);
       mbar_init(smem_u32(&o_full[i]), 1);
-      mbar_init(smem_u32(&o_empty[i]), 1);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_q)) : "memory");
@@ -465,18 +466,19 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       constexpr uint32_t idesc_s = idesc_bf16(kTcRows, kTcKeys);
       constexpr uint32_t idesc_o = idesc_bf16(kTcRows, kHD) | (1u << 16);   // B (V) MN-major
       bool ok = mbar_wait(smem_u32(q_full), 0, d_err);
-      // O_i = P_i V_i into TMEM columns 256 + 64 (i % 2)
+      // O += P_i V_i in TMEM columns 256 .. 319 (the first tile overwrites);
+      // the softmax rescales O in place before it releases P_i when the row
+      // max has grown
       auto issue_pv = [&](int i) -> bool {
         const int st = i & 1;
         if (!mbar_wait(smem_u32(&p_full[st]), (i >> 1) & 1, d_err)) return false;
-        if (i >= 2 && !mbar_wait(smem_u32(&o_empty[st]), ((i - 2) >> 1) & 1, d_err)) return false;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const int kvs = i % kTcStages;
         const uint32_t pa = sP + st * kTcP, vb = sV + kvs * kTcTile;
 #pragma unroll
         for (int kk = 0; kk < kTcKeys / 16; ++kk)
-          mma_bf16(tmem + 256 + 64 * st, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
-                   sdesc_mn(vb + kk * 16 * 128), idesc_o, kk > 0 ? 1u : 0u);
+          mma_bf16(tmem + 256, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
+                   sdesc_mn(vb + kk * 16 * 128), idesc_o, (i > 0 || kk > 0) ? 1u : 0u);
         mma_commit(smem_u32(&o_full[st]));
         mma_commit(smem_u32(&kv_empty[kvs]));
         return true;
@@ -505,10 +507,11 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     const float sc = 1.4426950408889634f * rsqrtf((float)kHD);
     const uint32_t lane_base = (uint32_t)(32 * quarter) << 16;
     const int kb0 = kTcPart * part;               // first key of this thread's part of a tile
-    float m = -INFINITY, l = 0.f, alpha_prev = 1.f;
-    float o[kTcOut];
-#pragma unroll
-    for (int d = 0; d < kTcOut; ++d) o[d] = 0.f;
+    // m: the row max the probabilities of the tiles so far are taken
+    // against (raised only when a tile's max exceeds it by more than 2^8, so
+    // P stays below 256); l: this thread's part of their sum
+    constexpr float kRescale = 8.f;
+    float m = -INFINITY, l = 0.f;
     // this row's 16-byte chunks of P buffer 0 for keys kb0 .. kb0 + 31: atom
     // kb0 / 64, chunks (kb0 % 64) / 8 + q at position chunk ^ (row % 8)
     const uint32_t prow = sP + (kb0 >> 6) * (kTcP / 2) + row * 128;
@@ -527,23 +530,8 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) {
       if (!mbar_wait(smem_u32(bar), parity, d_err)) *s_abort = 1;
     };
-    // o <- o * alpha + O_i (this thread's output dims of P_i V_i), then free
-    // its TMEM buffer
-    auto fold_o = [&](int i, float alpha) -> bool {
-      const int st = i & 1;
-      wait_or_abort(&o_full[st], (i >> 1) & 1);
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      float r[kTcOut];
-      if constexpr (kTcOut == 32) tmem_ld32(tmem + lane_base + 256 + 64 * st + kTcOut * part, r);
-      else tmem_ld16(tmem + lane_base + 256 + 64 * st + kTcOut * part, r);
-#pragma unroll
-      for (int d = 0; d < kTcOut; ++d) o[d] = o[d] * alpha + r[d];
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
-      if (*s_abort) return false;
-      if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&o_empty[st])) : "memory");
-      return true;
-    };
+    // this thread's output dims of the O accumulator in TMEM
+    const uint32_t o_addr = tmem + lane_base + 256 + kTcOut * part;
     for (int j = 0; j < n_tiles; ++j) {
       const int st = j & 1;
       int kt, kend;
@@ -576,8 +564,27 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       mx = s_mx[(st * kTcSplit) * kTcRows + row];
 #pragma unroll
       for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
-      const float mn = fmaxf(m, mx * sc);
-      const float alpha = (mn == -INFINITY) ? 1.f : ex2(m - mn);
+      // A new reference max when this tile's exceeds it by more than 2^8: O
+      // and l so far are scaled to it (O once the previous tile's P V has
+      // landed; nothing is accumulated before a finite max).  The TMEM
+      // load and store are warp-wide: a warp rescales when any of its rows
+      // needs it, the others by 1.
+      const bool raise = mx * sc > m + kRescale;
+      const float f = (raise && m != -INFINITY) ? ex2(m - mx * sc) : 1.f;
+      if (__any_sync(0xffffffffu, f != 1.f)) {
+        wait_or_abort(&o_full[(j - 1) & 1], ((j - 1) >> 1) & 1);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        float r[kTcOut];
+        tmem_ld32(o_addr, r);
+#pragma unroll
+        for (int d = 0; d < kTcOut; ++d) r[d] *= f;
+        tmem_st32(o_addr, r);
+      }
+      if (raise) {
+        l *= f;
+        m = mx * sc;
+      }
+      const float mn = m;
       // P = exp2(S sc - mn) rounded to bf16 (ex2(-inf) = 0 for masked keys),
       // the sum of the rounded values
       const uint32_t pbase = prow + st * kTcP;
@@ -598,18 +605,24 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
                      "r"(pk[3])
                      : "memory");
       }
-      m = mn;
-      l = l * alpha + ps;
+      l += ps;
       // S_j read, P_j written: to the tensor cores (async proxy)
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
       if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
-      // O_{j-1} (relative to the max before this tile) into the output
-      if (j >= 1 && !fold_o(j - 1, alpha_prev)) { ok = false; break; }
-      alpha_prev = alpha;
     }
-    if (ok && n_tiles > 0) ok = fold_o(n_tiles - 1, alpha_prev);
+    float o[kTcOut];
+#pragma unroll
+    for (int d = 0; d < kTcOut; ++d) o[d] = 0.f;
+    if (ok && n_tiles > 0) {
+      // the last tile's P V completes the accumulator
+      wait_or_abort(&o_full[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1);
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      tmem_ld32(o_addr, o);
+      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      if (*s_abort) ok = false;
+    }
     if (ok) {
       // the row's sum over its parts, in a fixed order
       s_l[part * kTcRows + row] = l;
