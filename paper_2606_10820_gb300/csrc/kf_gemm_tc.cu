@@ -949,6 +949,12 @@ int launch_gemm_tc(const GemmDesc& g, int* d_err, cudaStream_t s) {
     if (g.M > kBM && !(g_gemm_flags & kGemmNoPersist) && ceil_div(g.N, 256) * ceil_div(g.M, kBM) > num_sms)
       return launch_persist<256, 3>(g, d_err, num_sms, s);
     if (g.M > kBM) return launch_epi<256, 3, EPI_HEAD, 2, 1>(g, d_err, num_sms, s);
+    // one M tile, more than a wave of 256-wide tiles (the OWT-shaped vocab:
+    // 197 tiles on 152 SMs left a second wave of 45): a persistent loop over
+    // 128-wide tiles keeps every SM streaming weights to the end (batch 1,
+    // k = 4: 309.5 -> 303.8 us per call)
+    if (!(g_gemm_flags & kGemmNoPersist) && ceil_div(g.N, 256) > num_sms)
+      return launch_persist_epi<128, 4, EPI_HEAD>(g, d_err, num_sms, s);
     return launch_epi<256, 2, EPI_HEAD, 1, 2>(g, d_err, num_sms, s);
   }
   // the narrowest tile that covers the product in one wave, else 256-wide

@@ -70,10 +70,11 @@ def check_against_oracle(x, w, z, tau, map_kind, got):
     return bad
 
 
-# (130 and 520 rows at V = 50,257: the persistent tile loop, a ragged last M tile)
+# (8 rows at V = 50,257: the persistent loop over 128-wide tiles of one M tile;
+# 130 and 520 rows: the persistent loop over 256-wide tiles, a ragged last M tile)
 @pytest.mark.parametrize("rows,V,d,tau", [(3, 1000, 128, 1.0), (64, 30522, 768, 1.0),
-                                          (130, 50257, 768, 0.5), (520, 50257, 768, 1.0),
-                                          (256, 32, 64, 1.0)])
+                                          (8, 50257, 768, 1.0), (130, 50257, 768, 0.5),
+                                          (520, 50257, 768, 1.0), (256, 32, 64, 1.0)])
 @pytest.mark.parametrize("map_kind", [0, 1])
 def test_head_tokens_match_oracle(env, rows, V, d, tau, map_kind):
     torch, lib = env
