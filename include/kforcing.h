@@ -235,7 +235,9 @@ int kf_sync(kf_ctx* ctx);
  * graph with an event record node on each side of every launch (launches in
  * order, without programmatic dependent launch).  ms_per_kind[i] and launches_per_kind[i]
  * (arrays of KF_KIND_COUNT, host) receive the summed device time and launch
- * count per kernel kind.  Synchronises.
+ * count per kernel kind.  Synchronises.  The step's first kernel (row maps,
+ * pending-token embeddings and noise features in one launch) is counted under
+ * KF_KIND_EMBED; KF_KIND_ROWMAP stays at zero launches.
  */
 #define KF_KIND_ROWMAP 0
 #define KF_KIND_EMBED 1

@@ -377,16 +377,13 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
   const int kz = mtp ? 1 : k;                      // noise rows per sequence
   const int S = P + kz, R = B * S, nout = k > 0 ? k : 1, nh = mtp ? B : B * nout;
   c->skinny = use_skinny(c, R);
-  prof_begin(c, KF_KIND_ROWMAP);
-  launch_rowmap(B, P, kz, c->d_len, c->row_seq, c->row_pos, c->noise_map, c->head_map, s);
-  prof_end(c);
+  // row maps, pending-token embeddings and noise features: one launch
   prof_begin(c, KF_KIND_EMBED);
-  launch_embed_pending(c->bf16, B, P, kz, c->d_pending, c->pend_stride, c->tok_emb, c->pos_emb,
-                       c->row_pos, c->V, d, c->x, c->fused ? c->xn : nullptr,
-                       c->fused ? c->ss : nullptr, c->d_err, s);
-  if (k > 0)
-    launch_noise_feat(c->bf16, B * k, noise, c->noise_freq, c->tau_feat, c->cfg.noise_scale, d,
-                      c->nfeat, s);
+  launch_step_prologue(c->bf16, B, P, kz, c->d_len, c->d_pending, c->pend_stride, c->tok_emb,
+                       c->pos_emb, c->V, d, c->x, c->fused ? c->xn : nullptr,
+                       c->fused ? c->ss : nullptr, c->d_err, c->row_seq, c->row_pos, c->noise_map,
+                       c->head_map, k > 0 ? B * k : 0, noise, c->noise_freq, c->tau_feat,
+                       c->cfg.noise_scale, c->nfeat, s);
   prof_end(c);
   if (k > 0) {
     // h_z = NoiseEnc(z): W2 . gelu(W1 s(z, tau) + b1) + b2, written into the noise rows

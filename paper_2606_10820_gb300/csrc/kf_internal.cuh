@@ -499,19 +499,20 @@ int* op_error_word(cudaStream_t s);
 void set_global_error(const std::string& msg);
 
 // elementwise / bookkeeping kernels
-void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
-                   int32_t* noise_map, int32_t* head_map, cudaStream_t s);
-// xb / ss: bf16 copy and per-64-column sums of squares (fused RMSNorm), or NULL
-void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
-                          const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
-                          int V, int d, float* x, void* xb, float* ss, int* d_err, cudaStream_t s);
+// the first kernel of a decode step: the row maps, the embedding of the B*P
+// pending rows (xb / ss: bf16 copy and per-64-column sums of squares for the
+// fused RMSNorm, or NULL) and the features of n_noise noise values
+void launch_step_prologue(bool bf16, int B, int P, int kz, const int32_t* d_len, const int32_t* pending,
+                          int pend_stride, const void* tok_emb, const float* pos_emb, int V, int d,
+                          float* x, void* xb, float* ss, int* d_err, int32_t* row_seq, int32_t* row_pos,
+                          int32_t* noise_map, int32_t* head_map, int n_noise, const float* noise,
+                          const float* freq, const float* tau_feat, float scale, void* feat,
+                          cudaStream_t s);
 void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
                          const float* pos_emb, const int32_t* row_pos, int V, int d, float* x,
                          void* xb, float* ss, int* d_err, cudaStream_t s);
 void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, size_t total,
                        cudaStream_t s);
-void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, const float* tau_feat,
-                       float scale, int d, void* feat, cudaStream_t s);
 void launch_rmsnorm(bool bf16, int R, const int32_t* row_map, const float* x, int d,
                     const float* g, float eps, void* out, cudaStream_t s);
 void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,

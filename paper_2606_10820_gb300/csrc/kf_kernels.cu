@@ -8,52 +8,19 @@
 
 namespace kf {
 
-// ------------------------------------------------------------------ rows
-// Alg. 1 row layout per sequence b: P pending tokens at positions
-// c_b .. c_b+P-1, then k noise slots at c_b+P .. c_b+P+k-1.
-__global__ void k_rowmap(int B, int P, int k, const int32_t* __restrict__ len,
-                         int32_t* row_seq, int32_t* row_pos, int32_t* noise_map,
-                         int32_t* head_map) {
-  // the step's later kernels launch only after this wait (pdl_wait triggers
-  // them): each may read the cached lengths before its own dependency wait
-  // (they change only at the step's commit, and the previous step's commit
-  // is complete once this wait returns)
-  pdl_wait();
-  int r = blockIdx.x * blockDim.x + threadIdx.x;
-  int S = P + k;
-  if (r < B * S) {
-    int b = r / S, i = r - b * S;
-    row_seq[r] = b;
-    row_pos[r] = len[b] + i;
-  }
-  if (k > 0 && r < B * k) {
-    int b = r / k, j = r - b * k;
-    noise_map[r] = b * S + P + j;
-    head_map[r] = b * S + P + j;
-  }
-  if (k == 0 && r < B) head_map[r] = r * S + P - 1;
-}
-
-void launch_rowmap(int B, int P, int k, const int32_t* d_len, int32_t* row_seq, int32_t* row_pos,
-                   int32_t* noise_map, int32_t* head_map, cudaStream_t s) {
-  int n = B * (P + k);
-  kf_launch(k_rowmap, dim3(ceil_div(n, 128)), dim3(128), 0, s, B, P, k, d_len, row_seq, row_pos, noise_map, head_map);
-}
-
 // ------------------------------------------------------------ embeddings
-// x[r] = E[tok] (+ pos_emb[pos]).  With the fused RMSNorm (xb != NULL) the
-// row is also written as bf16 into xb and the sum of squares of each of its
+// x[r] = E[tok] (+ pos_row).  With the fused RMSNorm (xb != NULL) the row is
+// also written as bf16 into xb and the sum of squares of each of its
 // 64-column slots into ss[r][d/64] (warp partials over 32 columns, then the
-// pair of a slot added in order).  The token id and its embedding row do not
-// depend on the step's earlier kernels: a thread loads its (at most
-// kEmbedPer) columns before the dependency wait, all loads in flight at once.
+// pair of a slot added in order).  A thread loads its (at most kEmbedPer)
+// columns of the embedding row before the dependency wait, all loads in
+// flight at once (a no-op wait where the caller has already waited).
 constexpr int kEmbedThreads = 128;
 constexpr int kEmbedPer = 8;           // d <= 1024 kept in registers
 
 template <typename TA>
-__device__ void embed_row(int r, int tok, const int32_t* __restrict__ row_pos, const TA* __restrict__ emb,
-                          const float* __restrict__ pos_emb, int V, int d, float* x, TA* xb,
-                          float* ss, int* d_err) {
+__device__ void embed_row(int r, int tok, const float* __restrict__ pos_row, const TA* __restrict__ emb,
+                          int V, int d, float* x, TA* xb, float* ss, int* d_err) {
   __shared__ float part[128];          // d <= 4096
   const bool good = tok >= 0 && tok < V;
   const TA* e = emb + (size_t)(good ? tok : 0) * d;
@@ -68,7 +35,6 @@ __device__ void embed_row(int r, int tok, const int32_t* __restrict__ row_pos, c
   pdl_wait();
   if (!good && threadIdx.x == 0) atomicOr(d_err, kErrBadToken);
   float* o = x + (size_t)r * d;
-  const float* p = pos_emb ? pos_emb + (size_t)row_pos[r] * d : nullptr;
   for (int c0 = threadIdx.x - lane, j = 0; c0 < d; c0 += kEmbedThreads, ++j) {
     const int c = c0 + lane;
     float w = 0.f;
@@ -81,7 +47,7 @@ __device__ void embed_row(int r, int tok, const int32_t* __restrict__ row_pos, c
       } else {
         base = good ? to_f(e[c]) : 0.f;
       }
-      w = good ? base + (p ? p[c] : 0.f) : 0.f;
+      w = good ? base + (pos_row ? pos_row[c] : 0.f) : 0.f;
       o[c] = w;
       if (xb) xb[(size_t)r * d + c] = from_f<TA>(w);
     }
@@ -98,40 +64,15 @@ __device__ void embed_row(int r, int tok, const int32_t* __restrict__ row_pos, c
   }
 }
 
-// the pending ids were written by the previous step's commit, which has
-// completed before any kernel after the step's first one launches
-template <typename TA>
-__global__ void __launch_bounds__(kEmbedThreads)
-k_embed_pending(int P, int k, const int32_t* __restrict__ pending, int pend_stride,
-                const TA* __restrict__ emb, const float* __restrict__ pos_emb,
-                const int32_t* __restrict__ row_pos, int V, int d, float* x,
-                TA* xb, float* ss, int* d_err) {
-  int b = blockIdx.x / P, i = blockIdx.x - b * P;
-  int r = b * (P + k) + i;
-  embed_row<TA>(r, pending[b * pend_stride + i], row_pos, emb, pos_emb, V, d, x, xb, ss, d_err);
-}
-
-// the row tokens are copied from the host before the launch
+// the row tokens and positions are copied from the host before the launch
 template <typename TA>
 __global__ void __launch_bounds__(kEmbedThreads)
 k_embed_tokens(const int32_t* __restrict__ row_tok, const TA* __restrict__ emb,
                const float* __restrict__ pos_emb, const int32_t* __restrict__ row_pos,
                int V, int d, float* x, TA* xb, float* ss, int* d_err) {
   int r = blockIdx.x;
-  embed_row<TA>(r, row_tok[r], row_pos, emb, pos_emb, V, d, x, xb, ss, d_err);
-}
-
-void launch_embed_pending(bool bf16, int B, int P, int k, const int32_t* pending, int pend_stride,
-                          const void* tok_emb, const float* pos_emb, const int32_t* row_pos,
-                          int V, int d, float* x, void* xb, float* ss, int* d_err, cudaStream_t s) {
-  if (B * P == 0) return;
-  if (bf16)
-    kf_launch(k_embed_pending<__nv_bfloat16>, dim3(B * P), dim3(kEmbedThreads), 0, s, P, k, pending,
-              pend_stride, (const __nv_bfloat16*)tok_emb, pos_emb, row_pos, V, d, x,
-              (__nv_bfloat16*)xb, ss, d_err);
-  else
-    kf_launch(k_embed_pending<float>, dim3(B * P), dim3(kEmbedThreads), 0, s, P, k, pending, pend_stride,
-              (const float*)tok_emb, pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
+  embed_row<TA>(r, row_tok[r], pos_emb ? pos_emb + (size_t)row_pos[r] * d : nullptr, emb, V, d, x,
+                xb, ss, d_err);
 }
 
 void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* tok_emb,
@@ -145,6 +86,92 @@ void launch_embed_tokens(bool bf16, int R, const int32_t* row_tok, const void* t
   else
     kf_launch(k_embed_tokens<float>, dim3(R), dim3(kEmbedThreads), 0, s, row_tok, (const float*)tok_emb,
               pos_emb, row_pos, V, d, x, (float*)xb, ss, d_err);
+}
+
+// --------------------------------------------------------- step prologue
+// The first kernel of a decode step runs three independent jobs, one per
+// block range, so that no kernel boundary separates them:
+//  - blocks [0, B*P): the embedding of pending token i of sequence b into
+//    row b*S + i at position c_b + i (Alg. 1 row layout: P pending tokens at
+//    c_b .. c_b+P-1, then kz noise slots at c_b+P .. c_b+P+kz-1, S = P + kz);
+//  - the next map_blocks blocks: the row maps (sequence and position of each
+//    row, the noise rows that NoiseEnc writes, the rows the LM head reads);
+//  - the rest: the noise features of the n_noise noise values (Table 4:
+//    sinusoidal encodings of z and of tau, summed; [cos | sin] halves,
+//    freq[t] = exp(-ln(1e4) t / (d/2)), the argument (scale * z) * freq[t]
+//    formed in fp32 in that order (the oracle's arithmetic), its cosine
+//    and sine from sincosf; tau's encoding is the same for every row and is
+//    formed once per context).
+// Every block first waits for the previous step: its commit wrote the
+// lengths and the pending ids.  The wait also releases the step's later
+// kernels, which may then read the lengths before their own waits (they
+// change only at a commit).
+template <typename TA>
+__global__ void __launch_bounds__(kEmbedThreads)
+k_step_prologue(int B, int P, int kz, int map_blocks, const int32_t* __restrict__ len,
+                const int32_t* __restrict__ pending, int pend_stride, const TA* __restrict__ emb,
+                const float* __restrict__ pos_emb, int V, int d, float* x, TA* xb, float* ss,
+                int* d_err, int32_t* row_seq, int32_t* row_pos, int32_t* noise_map, int32_t* head_map,
+                int n_noise, const float* __restrict__ noise, const float* __restrict__ freq,
+                const float* __restrict__ tau_feat, float scale, TA* __restrict__ feat) {
+  pdl_wait();
+  const int S = P + kz;
+  int blk = blockIdx.x;
+  if (blk < B * P) {
+    const int b = blk / P, i = blk - b * P;
+    const int pos = len[b] + i;
+    embed_row<TA>(b * S + i, pending[b * pend_stride + i],
+                  pos_emb ? pos_emb + (size_t)pos * d : nullptr, emb, V, d, x, xb, ss, d_err);
+    return;
+  }
+  blk -= B * P;
+  if (blk < map_blocks) {
+    const int r = blk * kEmbedThreads + threadIdx.x;
+    if (r < B * S) {
+      const int b = r / S, i = r - b * S;
+      row_seq[r] = b;
+      row_pos[r] = len[b] + i;
+    }
+    if (kz > 0 && r < B * kz) {
+      const int b = r / kz, j = r - b * kz;
+      noise_map[r] = b * S + P + j;
+      head_map[r] = b * S + P + j;
+    }
+    if (kz == 0 && r < B) head_map[r] = r * S + P - 1;
+    return;
+  }
+  blk -= map_blocks;
+  const int half = d / 2;
+  const int idx = blk * kEmbedThreads + threadIdx.x;
+  if (idx >= n_noise * half) return;
+  const int r = idx / half, t = idx - r * half;
+  const float ang = __fmul_rn(__fmul_rn(scale, noise[r]), freq[t]);
+  float sz, cz;
+  sincosf(ang, &sz, &cz);
+  feat[(size_t)r * d + t] = from_f<TA>(cz + tau_feat[t]);
+  feat[(size_t)r * d + half + t] = from_f<TA>(sz + tau_feat[half + t]);
+}
+
+void launch_step_prologue(bool bf16, int B, int P, int kz, const int32_t* d_len, const int32_t* pending,
+                          int pend_stride, const void* tok_emb, const float* pos_emb, int V, int d,
+                          float* x, void* xb, float* ss, int* d_err, int32_t* row_seq, int32_t* row_pos,
+                          int32_t* noise_map, int32_t* head_map, int n_noise, const float* noise,
+                          const float* freq, const float* tau_feat, float scale, void* feat,
+                          cudaStream_t s) {
+  const int map_blocks = ceil_div(B * (P + kz), kEmbedThreads);
+  const int noise_blocks = ceil_div(n_noise * (d / 2), kEmbedThreads);
+  const dim3 grid(B * P + map_blocks + noise_blocks);
+  if (grid.x == 0) return;
+  if (bf16)
+    kf_launch(k_step_prologue<__nv_bfloat16>, grid, dim3(kEmbedThreads), 0, s, B, P, kz, map_blocks,
+              d_len, pending, pend_stride, (const __nv_bfloat16*)tok_emb, pos_emb, V, d, x,
+              (__nv_bfloat16*)xb, ss, d_err, row_seq, row_pos, noise_map, head_map, n_noise, noise,
+              freq, tau_feat, scale, (__nv_bfloat16*)feat);
+  else
+    kf_launch(k_step_prologue<float>, grid, dim3(kEmbedThreads), 0, s, B, P, kz, map_blocks, d_len,
+              pending, pend_stride, (const float*)tok_emb, pos_emb, V, d, x, (float*)xb, ss, d_err,
+              row_seq, row_pos, noise_map, head_map, n_noise, noise, freq, tau_feat, scale,
+              (float*)feat);
 }
 
 // w[r][c] *= g[(r / rows_per_layer) * cols + c]: folds RMSNorm gains into the
@@ -165,43 +192,6 @@ void launch_scale_cols(float* w, const float* g, int rows_per_layer, int cols, s
   if (total == 0) return;
   int blocks = (int)std::min<size_t>((total + 255) / 256, 65535);
   k_scale_cols<<<blocks, 256, 0, s>>>(w, g, rows_per_layer, cols, total);
-}
-
-// ------------------------------------------------------- noise features
-// Sinusoidal encoding of z and of tau (Table 4), summed; argument
-// scale * u * freq[t], freq[t] = exp(-ln(1e4) t / (d/2)); [cos | sin].
-// The angle (up to scale radians) is formed and reduced modulo 2 pi in fp64
-// (a few DFMAs), then sincosf runs on the reduced fp32 angle: the feature is
-// accurate to fp32 rounding without fp64 transcendentals.
-// tau_feat: the temperature's encoding [cos | sin] of scale * tau * freq, the
-// same for every row (formed once per context).  The noise's angle is
-// (scale * z) * freq in fp32, in that order (the oracle's arithmetic), and
-// its cosine and sine come from sincosf (full argument reduction).
-template <typename TA>
-__global__ void k_noise_feat(int n, const float* __restrict__ noise, const float* __restrict__ freq,
-                             const float* __restrict__ tau_feat, float scale, int d, TA* __restrict__ feat) {
-  pdl_wait();
-  int half = d / 2;
-  int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= n * half) return;
-  int r = idx / half, t = idx - r * half;
-  const float ang = __fmul_rn(__fmul_rn(scale, noise[r]), freq[t]);
-  float sz, cz;
-  sincosf(ang, &sz, &cz);
-  feat[(size_t)r * d + t] = from_f<TA>(cz + tau_feat[t]);
-  feat[(size_t)r * d + half + t] = from_f<TA>(sz + tau_feat[half + t]);
-}
-
-void launch_noise_feat(bool bf16, int n, const float* noise, const float* freq, const float* tau_feat,
-                       float scale, int d, void* feat, cudaStream_t s) {
-  if (n == 0) return;
-  int tot = n * (d / 2);
-  if (bf16)
-    kf_launch(k_noise_feat<__nv_bfloat16>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau_feat,
-              scale, d, (__nv_bfloat16*)feat);
-  else
-    kf_launch(k_noise_feat<float>, dim3(ceil_div(tot, 256)), dim3(256), 0, s, n, noise, freq, tau_feat, scale, d,
-              (float*)feat);
 }
 
 // --------------------------------------------------------------- RMSNorm
