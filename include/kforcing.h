@@ -237,7 +237,9 @@ int kf_sync(kf_ctx* ctx);
  * (arrays of KF_KIND_COUNT, host) receive the summed device time and launch
  * count per kernel kind.  Synchronises.  The step's first kernel (row maps,
  * pending-token embeddings and noise features in one launch) is counted under
- * KF_KIND_EMBED; KF_KIND_ROWMAP stays at zero launches.
+ * KF_KIND_EMBED, and the step's commit is taken by the token selection
+ * (KF_KIND_HEAD_SELECT); KF_KIND_ROWMAP and KF_KIND_COMMIT stay at zero
+ * launches.
  */
 #define KF_KIND_ROWMAP 0
 #define KF_KIND_EMBED 1

@@ -423,13 +423,15 @@ static void enqueue_step(kf_ctx* c, int B, int P, int k, const float* noise) {
     eh.nchunk = c->nchunk;
     gemm(c, KF_KIND_GEMM_HEAD, nh, c->V_pad, d, c->head_in, d, c->w_head, d, eh);
   }
+  // the noise -> token map, which also commits the step (the emitted tokens
+  // become the pending ids, the lengths grow by P)
+  StepCommit cm;
+  cm.pending = c->d_pending; cm.pend_stride = c->pend_stride; cm.len = c->d_len; cm.P = P;
+  cm.nout = nout;
   prof_begin(c, KF_KIND_HEAD_SELECT);
   launch_head_select(c->bf16, B * nout, c->rec, c->nchunk, c->head_in, d, mtp ? c->w_mtp : c->w_head,
                      c->V, 1.0f / c->cfg.tau, c->cfg.map_kind, noise, c->tokens, mtp ? B : 0,
-                     (size_t)c->V_pad * d, c->d_err, s);
-  prof_end(c);
-  prof_begin(c, KF_KIND_COMMIT);
-  launch_commit(B, P, k, c->tokens, c->d_pending, c->pend_stride, c->d_len, s);
+                     (size_t)c->V_pad * d, c->d_err, cm, s);
   prof_end(c);
 }
 

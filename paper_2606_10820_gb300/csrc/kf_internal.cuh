@@ -520,6 +520,16 @@ void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
                         const int32_t* row_pos, const float* cos_t, const float* sin_t, float* q,
                         void* kv, int layer, int n_pages, const int32_t* page_table, int max_pages,
                         int* d_err, cudaStream_t s);
+// A decode step's commit, taken by the token selection: token b nout + j
+// becomes pending id j of sequence b (pending[b pend_stride + j]) and len[b]
+// grows by P.  pending == NULL: tokens only.
+struct StepCommit {
+  int32_t* pending = nullptr;
+  int pend_stride = 0;
+  int32_t* len = nullptr;
+  int P = 0;
+  int nout = 1;
+};
 // mtp_rows = B > 0: n_rows = B k blocks in head-major order, head j's weights
 // at w_head + j head_stride (elements); 0: one block per row of head_in.
 // err: the call's device error word (or NULL); when an earlier kernel set
@@ -527,8 +537,6 @@ void launch_rope_append(bool bf16, int R, const void* qkv, int d, int H, int hd,
 void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
                         int d, const void* w_head, int V, float inv_tau, int map_kind,
                         const float* noise, int32_t* tokens, int mtp_rows, size_t head_stride,
-                        const int* err, cudaStream_t s);
-void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
-                   int32_t* d_len, cudaStream_t s);
+                        const int* err, const StepCommit& cm, cudaStream_t s);
 
 }  // namespace kf

@@ -364,12 +364,27 @@ template <> __device__ __forceinline__ double chunk_scale<double>(float m, float
   return exp((double)m - (double)M);
 }
 
+// Token zrow = b nout + j is written to tokens and, in a decode step, the
+// step's commit (C <- [C; C_x], App. C.1 fixed stride) is taken here: it
+// becomes pending token j of sequence b, and sequence b's block j = 0 adds the
+// P newly cached tokens to its length.  Every kernel that reads the lengths or
+// the pending ids in this step has completed (the dependency wait), and the
+// next step's first kernel reads them only after its own wait.
+__device__ __forceinline__ void emit_token(int32_t* tokens, int zrow, int tok, const StepCommit& cm) {
+  tokens[zrow] = tok;
+  if (cm.pending) {
+    const int b = zrow / cm.nout, j = zrow - b * cm.nout;
+    cm.pending[(size_t)b * cm.pend_stride + j] = tok;
+    if (j == 0) cm.len[b] += cm.P;
+  }
+}
+
 template <typename TA>
 __global__ void __launch_bounds__(kSelThreads)
 k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restrict__ head_in, int d,
               const TA* __restrict__ w_head_all, int V, float inv_tau, int map_kind,
               const float* __restrict__ noise, int32_t* __restrict__ tokens, int mtp_rows,
-              size_t head_stride, const int* __restrict__ err) {
+              size_t head_stride, const int* __restrict__ err, StepCommit cm) {
   pdl_wait();
   // one block per mapped row; MTP (mtp_rows = B > 0): block j B + b is head j
   // of sequence b (records in that order), hidden row b, weights w_head + j
@@ -388,7 +403,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   // Every earlier kernel has completed (pdl_wait), so all threads read the
   // same value.
   if (err && *err) {
-    if (threadIdx.x == 0) tokens[zrow] = -1;
+    if (threadIdx.x == 0) emit_token(tokens, zrow, -1, cm);
     return;
   }
   // the inverse-CDF sums: fp32 for the bf16 model (its logits carry bf16
@@ -450,7 +465,7 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
   }
   __syncthreads();
   if (map_kind == KF_MAP_ARGMAX) {
-    if (t == 0) tokens[zrow] = s_redi[0];
+    if (t == 0) emit_token(tokens, zrow, s_redi[0], cm);
     return;
   }
   const float M = s_M;
@@ -580,40 +595,22 @@ k_head_select(const HeadRec* __restrict__ rec_all, int nchunk, const TA* __restr
     if (hit) tok = cstar * kChunk + (__ffs(hit) - 1);
     else if (pos) tok = cstar * kChunk + (31 - __clz(pos));
     else tok = min(V - 1, cstar * kChunk + 31);
-    tokens[zrow] = tok;
+    emit_token(tokens, zrow, tok, cm);
   }
 }
 
 void launch_head_select(bool bf16, int n_rows, const HeadRec* rec, int nchunk, const void* head_in,
                         int d, const void* w_head, int V, float inv_tau, int map_kind,
                         const float* noise, int32_t* tokens, int mtp_rows, size_t head_stride,
-                        const int* err, cudaStream_t s) {
+                        const int* err, const StepCommit& cm, cudaStream_t s) {
   if (n_rows == 0) return;
   if (bf16)
     kf_launch(k_head_select<__nv_bfloat16>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk,
         (const __nv_bfloat16*)head_in, d, (const __nv_bfloat16*)w_head, V, inv_tau, map_kind,
-        noise, tokens, mtp_rows, head_stride, err);
+        noise, tokens, mtp_rows, head_stride, err, cm);
   else
     kf_launch(k_head_select<float>, dim3(n_rows), dim3(kSelThreads), 0, s, rec, nchunk, (const float*)head_in, d,
-        (const float*)w_head, V, inv_tau, map_kind, noise, tokens, mtp_rows, head_stride, err);
-}
-
-// ---------------------------------------------------------------- commit
-// C <- [C; C_x]: the P pending tokens are now cached; the emitted tokens
-// become the next step's pending tokens (App. C.1 fixed stride).
-__global__ void k_commit(int B, int P, int nout, const int32_t* __restrict__ tokens,
-                         int32_t* pending, int pend_stride, int32_t* len) {
-  pdl_wait();
-  int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= B) return;
-  for (int j = 0; j < nout; ++j) pending[b * pend_stride + j] = tokens[b * nout + j];
-  len[b] += P;
-}
-
-void launch_commit(int B, int P, int k, const int32_t* tokens, int32_t* pending, int pend_stride,
-                   int32_t* d_len, cudaStream_t s) {
-  int nout = k > 0 ? k : 1;
-  kf_launch(k_commit, dim3(ceil_div(B, 128)), dim3(128), 0, s, B, P, nout, tokens, pending, pend_stride, d_len);
+        (const float*)w_head, V, inv_tau, map_kind, noise, tokens, mtp_rows, head_stride, err, cm);
 }
 
 }  // namespace kf

@@ -73,7 +73,7 @@ static int head_tokens(int32_t rows, int32_t V, int32_t d, const void* x, const 
   if (!tc_gemm_supported(g)) return KF_E_ARG;
   if (launch_gemm_tc(g, err, s) != 0) return KF_E_CUDA;
   launch_head_select(true, rows, rec, nchunk, x, d, w_head, V, 1.0f / tau, map_kind, noise, tokens, 0, 0,
-                     err, s);
+                     err, StepCommit{}, s);
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
 }
 

@@ -288,16 +288,23 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
 }
 
 // ------------------------------------------------------------------ tcgen05
-// The same attention on the 5th-generation tensor cores.  A CTA takes 128
-// query rows of one (sequence, head) and walks the same key ranges in tiles
-// of 128 keys (each range's tiles start at its first key; keys past the
-// range's end are masked, so no key is counted twice):
-//   warp 0      TMA: Q once, then K and V tiles of [128 keys][64] bf16
-//               (128-byte swizzle) into a four-stage ring;
+// The same attention on the 5th-generation tensor cores.  A work item is 128
+// query rows of one (sequence, head); its key ranges are walked in tiles of
+// 128 keys (each range's tiles start at its first key; keys past the range's
+// end are masked, so no key is counted twice).  The kernel is persistent:
+// one CTA per SM takes items blockIdx.x, blockIdx.x + gridDim.x, ... (the
+// query tiles with the most keys first), and its roles run ahead across
+// items, so that the next item's copies and first products overlap this
+// item's last softmax tile and output:
+//   warp 0      TMA: an item's Q (once the previous item's last S product
+//               has read the Q buffer), then its K and V tiles of
+//               [128 keys][64] bf16 (128-byte swizzle) into a four-stage ring;
 //   warp 1      one thread issues tcgen05.mma: S_j = Q K_j^T (M = 128 rows,
 //               N = 128 keys, K = 64) into one of two TMEM buffers, and
 //               O += P_j V_j (M = 128, N = 64, K = 128 keys; V is the
-//               MN-major operand as loaded) into one TMEM accumulator;
+//               MN-major operand as loaded) into one TMEM accumulator, an
+//               item's first P V overwriting it once the softmax has read
+//               the previous item's O;
 //   warps 2..9  two threads per query row (TMEM lane), each with half of
 //               its keys and of its output (four threads measured 5 % slower:
 //               the per-tile chain of waits and barriers, not the arithmetic,
@@ -307,11 +314,13 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
 //               shared memory (K-major, swizzled: the A operand of P V).  m
 //               is raised only when a tile's max exceeds it by more than 2^8
 //               (P stays below 256); then O in TMEM and l are scaled to the
-//               new m before P_j is released.  At the end O / l is the row's
-//               output.
-// S of tile j + 1 is computed while the softmax works on tile j.  Every
-// wait is bounded; a wait that runs out sets the error word and ends the
-// CTA's loops.
+//               new m before P_j is released.  At the item's end O / l is
+//               the row's output.
+// Tiles are numbered across the CTA's items (g): S of tile g + 1 is computed
+// while the softmax works on tile g, and P V of tile g is issued after it
+// (an item's last P V right after its last S).
+// Every wait is bounded; a wait that runs out sets the error word and ends
+// the CTA's loops.
 namespace {
 constexpr int kTcRows = 128;
 constexpr int kTcKeys = 128;
@@ -328,15 +337,84 @@ constexpr uint32_t kTcP = kTcRows * kTcKeys * 2;      // 32 KB: one P tile (two 
 constexpr int kTcStages = 4;
 // [Q][K stages][V stages][P 2], the barriers and shared scalars (256 B),
 // then the row-max exchange [2 tiles][kTcSplit parts][128 rows] and the row
-// sums [kTcSplit][128]
+// sums [2 items][kTcSplit][128]
 constexpr size_t tc_smem_bytes() {
-  return 1024 + (1 + 2 * kTcStages) * (size_t)kTcTile + 2 * (size_t)kTcP + 256 + 3 * kTcSplit * 128 * 4;
+  return 1024 + (1 + 2 * kTcStages) * (size_t)kTcTile + 2 * (size_t)kTcP + 256 + 4 * kTcSplit * 128 * 4;
+}
+
+// The key ranges an item's 128 query rows open (the union over its rows:
+// the context prefix up to the largest context key, the block-1 and block-2
+// windows; an empty one has lo == hi), the smallest context key every valid
+// row sees, and the number of 128-key tiles.  Warp-collective: each lane
+// takes four rows.
+struct TileRanges {
+  int lo[3], hi[3], cmin, n;
+};
+
+__device__ __forceinline__ TileRanges tile_ranges(const TrainAttnArgs& a, int q0, int lane) {
+  int cmax = -1, cmin = 1 << 30, w1lo = 1 << 30, w1hi = 0, w2lo = 1 << 30, w2hi = 0;
+#pragma unroll
+  for (int i = 0; i < kTcRows / 32; ++i) {
+    const RowVis v = row_vis(a, q0 + lane + 32 * i);
+    if (v.ctx < 0) continue;
+    cmax = max(cmax, v.ctx);
+    cmin = min(cmin, v.ctx);
+    if (v.w1hi > v.w1lo) { w1lo = min(w1lo, v.w1lo); w1hi = max(w1hi, v.w1hi); }
+    if (v.w2hi > v.w2lo) { w2lo = min(w2lo, v.w2lo); w2hi = max(w2hi, v.w2hi); }
+  }
+  cmax = __reduce_max_sync(0xffffffffu, cmax);
+  cmin = __reduce_min_sync(0xffffffffu, cmin);
+  w1lo = __reduce_min_sync(0xffffffffu, w1lo);
+  w1hi = __reduce_max_sync(0xffffffffu, w1hi);
+  w2lo = __reduce_min_sync(0xffffffffu, w2lo);
+  w2hi = __reduce_max_sync(0xffffffffu, w2hi);
+  TileRanges r;
+  if (a.dense) {
+    r.lo[0] = 0; r.hi[0] = a.T;
+    r.lo[1] = r.hi[1] = r.lo[2] = r.hi[2] = 0;
+  } else {
+    r.lo[0] = 0; r.hi[0] = cmax + 1;                              // 0 when no valid row
+    r.lo[1] = w1lo; r.hi[1] = max(w1lo, w1hi);
+    r.lo[2] = w2lo; r.hi[2] = max(w2lo, w2hi);
+  }
+  r.cmin = cmin;
+  r.n = 0;
+#pragma unroll
+  for (int i = 0; i < 3; ++i) r.n += ceil_div(r.hi[i] - r.lo[i], kTcKeys);
+  return r;
+}
+
+// named barrier 1 over the softmax threads that also ORs a predicate over
+// them: every thread gets the same answer, so all leave a loop together
+__device__ __forceinline__ bool softmax_bar_or(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, 1, %2, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "n"(kTcSoftmax)
+      : "memory");
+  return r != 0;
+}
+
+// first key and range end of tile j of an item (constant indices only: the
+// ranges stay in registers)
+__device__ __forceinline__ void tile_at(const TileRanges& r, int j, int* lo, int* hi) {
+  *lo = 0; *hi = 0;
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    const int n = ceil_div(r.hi[i] - r.lo[i], kTcKeys);
+    if (j >= 0 && j < n) { *lo = r.lo[i] + j * kTcKeys; *hi = r.hi[i]; }
+    j -= n;
+  }
 }
 }  // namespace
 
 __global__ void __launch_bounds__(kTcThreads, 1)
 k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                     const __grid_constant__ CUtensorMap map_v, TrainAttnArgs a, int* d_err) {
+                     const __grid_constant__ CUtensorMap map_v, TrainAttnArgs a, int n_batch, int* d_err) {
   extern __shared__ __align__(1024) uint8_t tsm_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tsm_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(sm);
@@ -347,28 +425,46 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
   const uint32_t sP = smem_u32(Pp);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kPOff + 2 * kTcP);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;                      // [kTcStages]
+  uint64_t* q_empty = bars + 1;                      // the item's last S product done
+  uint64_t* kv_full = bars + 2;                      // [kTcStages]
   uint64_t* kv_empty = kv_full + kTcStages;          // [kTcStages]
   uint64_t* s_full = kv_empty + kTcStages;           // [2]
-  uint64_t* p_full = s_full + 2;                     // [2]: P_j written (and S_j read)
+  uint64_t* p_full = s_full + 2;                     // [2]: P_g written (and S_g read)
   uint64_t* o_full = p_full + 2;                     // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 2);
-  int* s_rng = reinterpret_cast<int*>(tmem_slot + 1);   // cmax, w1lo, w1hi, w2lo, w2hi, cmin
-  int* s_cnt = s_rng + 6;                                // tiles whose K/V the MMA has taken
-  volatile int* s_abort = s_cnt + 1;                     // a softmax thread's wait ran out
+  uint64_t* o_free = o_full + 2;                     // the item's O read out
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_free + 1);
+  int* s_cnt = reinterpret_cast<int*>(tmem_slot + 1);    // K/V tiles the MMA thread has taken
+  int* s_qcnt = s_cnt + 1;                               // Q tiles the MMA thread has taken
   float* s_mx = reinterpret_cast<float*>(sm + kPOff + 2 * kTcP + 256);         // [2][kTcSplit][128]
-  float* s_l = s_mx + 2 * kTcSplit * kTcRows;                                  // [kTcSplit][128]
+  float* s_l = s_mx + 2 * kTcSplit * kTcRows;                                  // [2][kTcSplit][128]
 
-  const int q0 = a.q_begin + blockIdx.x * kTcRows, h = blockIdx.y, b = blockIdx.z;
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int quarter = warp & 3;                 // softmax warps: TMEM lanes 32 quarter ..
   const int row = 32 * quarter + lane;          // this softmax thread's query row in the tile
   const int part = (warp - 2) >> 2;             // its keys kTcPart part .. and output dims kTcOut part ..
-  RowVis v{-1, 0, 0, 0, 0};
-  if (warp >= 2) v = row_vis(a, q0 + row);
+  const int n_qt = ceil_div(a.q_end - a.q_begin, kTcRows);
+  const int n_hb = a.H * n_batch;
+  const int n_items = n_qt * n_hb;
+  // the CTA's i-th item: rounds of gridDim.x items, walked forwards in even
+  // rounds and backwards in odd ones, so that each CTA's items add up to
+  // about the same number of tiles; -1 past the last
+  auto item_at = [&](int i) -> int {
+    const int P = gridDim.x, c = blockIdx.x;
+    const long long w = (long long)i * P + ((i & 1) ? P - 1 - c : c);
+    return w < n_items ? (int)w : -1;
+  };
+  // item w: query tile n_qt - 1 - w / n_hb (the most keys first), then head
+  // and sequence
+  auto item = [&](int w, int* q0, int* h, int* b) {
+    const int qt = w / n_hb, hb = w - qt * n_hb;
+    *q0 = a.q_begin + (n_qt - 1 - qt) * kTcRows;
+    *h = hb % a.H;
+    *b = hb / a.H;
+  };
 
   if (t == 0) {
     mbar_init(smem_u32(q_full), 1);
+    mbar_init(smem_u32(q_empty), 1);
     for (int i = 0; i < kTcStages; ++i) {
       mbar_init(smem_u32(&kv_full[i]), 1);
       mbar_init(smem_u32(&kv_empty[i]), 1);
@@ -378,13 +474,13 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
       mbar_init(smem_u32(&p_full[i]), 1);
       mbar_init(smem_u32(&o_full[i]), 1);
     }
+    mbar_init(smem_u32(o_free), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_q)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_k)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_v)) : "memory");
-    s_rng[0] = -1; s_rng[1] = 1 << 30; s_rng[2] = 0; s_rng[3] = 1 << 30; s_rng[4] = 0; s_rng[5] = 1 << 30;
     s_cnt[0] = 0;
-    *s_abort = 0;
+    s_qcnt[0] = 0;
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
@@ -396,109 +492,110 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = *tmem_slot;
-  // the key ranges of the CTA's rows (their union), and the context keys
-  // every valid row sees
-  if (warp >= 2 && v.ctx >= 0) {
-    atomicMax(&s_rng[0], v.ctx);
-    atomicMin(&s_rng[5], v.ctx);
-    if (v.w1hi > v.w1lo) { atomicMin(&s_rng[1], v.w1lo); atomicMax(&s_rng[2], v.w1hi); }
-    if (v.w2hi > v.w2lo) { atomicMin(&s_rng[3], v.w2lo); atomicMax(&s_rng[4], v.w2hi); }
-  }
-  __syncthreads();
-  // the CTA's key ranges: empty ones have lo == hi (no tiles)
-  int rlo[3], rhi[3];
-  const int nr = 3;
-  if (a.dense) {
-    rlo[0] = 0; rhi[0] = a.T;
-    rlo[1] = rhi[1] = rlo[2] = rhi[2] = 0;
-  } else {
-    rlo[0] = 0; rhi[0] = s_rng[0] + 1;                              // 0 when no valid row
-    rlo[1] = s_rng[1]; rhi[1] = max(s_rng[1], s_rng[2]);
-    rlo[2] = s_rng[3]; rhi[2] = max(s_rng[3], s_rng[4]);
-  }
-  const int cmin = s_rng[5];
-  // (constant indices only: the ranges stay in registers)
-  int n_tiles = 0;
-#pragma unroll
-  for (int i = 0; i < 3; ++i)
-    if (i < nr) n_tiles += ceil_div(rhi[i] - rlo[i], kTcKeys);
-  auto tile_at = [&](int j, int* lo, int* hi) {
-    *lo = 0; *hi = 0;
-#pragma unroll
-    for (int i = 0; i < 3; ++i) {
-      if (i < nr) {
-        const int n = ceil_div(rhi[i] - rlo[i], kTcKeys);
-        if (j >= 0 && j < n) { *lo = rlo[i] + j * kTcKeys; *hi = rhi[i]; }
-        j -= n;
-      }
-    }
-  };
   pdl_wait();
 
   if (warp == 0) {
-    if (lane == 0) {
-      mbar_expect_tx(smem_u32(q_full), kTcTile);
-      tma_load_4d(sQ, &map_q, smem_u32(q_full), 0, h, q0, b);
-      int issued = 0;
-      bool ok = true;
-      for (int j = 0; j < n_tiles; ++j) {
-        const int st = j % kTcStages;
-        if (j >= kTcStages && !mbar_wait(smem_u32(&kv_empty[st]), ((j / kTcStages) - 1) & 1, d_err)) {
-          ok = false;
-          break;
+    bool ok = true;
+    int g = 0, issued = 0, q_issued = 0, it = 0;
+    for (int w = item_at(0); ok && w >= 0; w = item_at(++it)) {
+      int q0, h, b;
+      item(w, &q0, &h, &b);
+      const TileRanges r = tile_ranges(a, q0, lane);
+      if (lane == 0) {
+        // the Q buffer is free once the previous item's last S product is done
+        if (it > 0 && !mbar_wait(smem_u32(q_empty), (it - 1) & 1, d_err)) ok = false;
+        if (ok) {
+          mbar_expect_tx(smem_u32(q_full), kTcTile);
+          tma_load_4d(sQ, &map_q, smem_u32(q_full), 0, h, q0, b);
+          q_issued = it + 1;
         }
-        int kt, kend;
-        tile_at(j, &kt, &kend);
-        mbar_expect_tx(smem_u32(&kv_full[st]), 2 * kTcTile);
-        tma_load_4d(sK + st * kTcTile, &map_k, smem_u32(&kv_full[st]), 0, h, kt, b);
-        tma_load_4d(sV + st * kTcTile, &map_v, smem_u32(&kv_full[st]), 0, h, kt, b);
-        issued = j + 1;
+        for (int j = 0; ok && j < r.n; ++j, ++g) {
+          const int st = g % kTcStages;
+          if (g >= kTcStages && !mbar_wait(smem_u32(&kv_empty[st]), ((g / kTcStages) - 1) & 1, d_err)) {
+            ok = false;
+            break;
+          }
+          int kt, kend;
+          tile_at(r, j, &kt, &kend);
+          mbar_expect_tx(smem_u32(&kv_full[st]), 2 * kTcTile);
+          tma_load_4d(sK + st * kTcTile, &map_k, smem_u32(&kv_full[st]), 0, h, kt, b);
+          tma_load_4d(sV + st * kTcTile, &map_v, smem_u32(&kv_full[st]), 0, h, kt, b);
+          issued = g + 1;
+        }
       }
-      if (!ok) {
-        // let the copies still in flight land before the CTA ends (bounded)
-        for (int j = *(volatile int*)s_cnt; j < issued; ++j)
-          mbar_wait(smem_u32(&kv_full[j % kTcStages]), (j / kTcStages) & 1, d_err);
-      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+    }
+    if (lane == 0 && !ok) {
+      // let the copies still in flight land before the CTA ends (bounded)
+      for (int j = *(volatile int*)s_cnt; j < issued; ++j)
+        mbar_wait(smem_u32(&kv_full[j % kTcStages]), (j / kTcStages) & 1, d_err);
+      if (q_issued > *(volatile int*)s_qcnt) mbar_wait(smem_u32(q_full), (q_issued - 1) & 1, d_err);
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idesc_s = idesc_bf16(kTcRows, kTcKeys);
-      constexpr uint32_t idesc_o = idesc_bf16(kTcRows, kHD) | (1u << 16);   // B (V) MN-major
-      bool ok = mbar_wait(smem_u32(q_full), 0, d_err);
-      // O += P_i V_i in TMEM columns 256 .. 319 (the first tile overwrites);
-      // the softmax rescales O in place before it releases P_i when the row
-      // max has grown
-      auto issue_pv = [&](int i) -> bool {
-        const int st = i & 1;
-        if (!mbar_wait(smem_u32(&p_full[st]), (i >> 1) & 1, d_err)) return false;
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const int kvs = i % kTcStages;
-        const uint32_t pa = sP + st * kTcP, vb = sV + kvs * kTcTile;
-#pragma unroll
-        for (int kk = 0; kk < kTcKeys / 16; ++kk)
-          mma_bf16(tmem + 256, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
-                   sdesc_mn(vb + kk * 16 * 128), idesc_o, (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(smem_u32(&o_full[st]));
-        mma_commit(smem_u32(&kv_empty[kvs]));
-        return true;
-      };
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const int st = j & 1;
-        if (!mbar_wait(smem_u32(&kv_full[j % kTcStages]), (j / kTcStages) & 1, d_err)) { ok = false; break; }
-        *(volatile int*)s_cnt = j + 1;
-        // S buffer st is free once the softmax has read S_{j-2}
-        if (j >= 2 && !mbar_wait(smem_u32(&p_full[st]), ((j - 2) >> 1) & 1, d_err)) { ok = false; break; }
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t kb = sK + (j % kTcStages) * kTcTile;
-#pragma unroll
-        for (int kk = 0; kk < kHD / 16; ++kk)
-          mma_bf16(tmem + kTcKeys * st, sdesc(sQ + kk * 32), sdesc(kb + kk * 32), idesc_s, kk > 0 ? 1u : 0u);
-        mma_commit(smem_u32(&s_full[st]));
-        if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+    constexpr uint32_t idesc_s = idesc_bf16(kTcRows, kTcKeys);
+    constexpr uint32_t idesc_o = idesc_bf16(kTcRows, kHD) | (1u << 16);   // B (V) MN-major
+    bool ok = true;
+    int g = 0, it = 0, o_items = 0;
+    int pv = -1;                  // the tile whose S is issued and whose P V is not
+    bool pv_first = false;        // ... the first tile of its item
+    // O += P_i V_i in TMEM columns 256 .. 319.  An item's first tile
+    // overwrites O once the softmax has read the previous item's O out; the
+    // softmax rescales O in place before it releases P_i when the row max
+    // has grown.
+    auto issue_pv = [&](int i, bool first) -> bool {
+      if (first) {
+        if (o_items > 0 && !mbar_wait(smem_u32(o_free), (o_items - 1) & 1, d_err)) return false;
+        ++o_items;
       }
-      if (ok && n_tiles > 0) issue_pv(n_tiles - 1);
+      const int st = i & 1;
+      if (!mbar_wait(smem_u32(&p_full[st]), (i >> 1) & 1, d_err)) return false;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const int kvs = i % kTcStages;
+      const uint32_t pa = sP + st * kTcP, vb = sV + kvs * kTcTile;
+#pragma unroll
+      for (int kk = 0; kk < kTcKeys / 16; ++kk)
+        mma_bf16(tmem + 256, sdesc(pa + (kk >> 2) * (kTcP / 2) + (kk & 3) * 32),
+                 sdesc_mn(vb + kk * 16 * 128), idesc_o, (!first || kk > 0) ? 1u : 0u);
+      mma_commit(smem_u32(&o_full[st]));
+      mma_commit(smem_u32(&kv_empty[kvs]));
+      return true;
+    };
+    for (int w = item_at(0); ok && w >= 0; w = item_at(++it)) {
+      int q0, h, b;
+      item(w, &q0, &h, &b);
+      const TileRanges r = tile_ranges(a, q0, lane);
+      if (lane == 0) {
+        ok = mbar_wait(smem_u32(q_full), it & 1, d_err);
+        if (ok) *(volatile int*)s_qcnt = it + 1;
+        for (int j = 0; ok && j < r.n; ++j, ++g) {
+          const int st = g & 1;
+          if (!mbar_wait(smem_u32(&kv_full[g % kTcStages]), (g / kTcStages) & 1, d_err)) { ok = false; break; }
+          *(volatile int*)s_cnt = g + 1;
+          // S buffer st is free once the softmax has read S_{g-2}
+          if (g >= 2 && !mbar_wait(smem_u32(&p_full[st]), ((g - 2) >> 1) & 1, d_err)) { ok = false; break; }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t kb = sK + (g % kTcStages) * kTcTile;
+#pragma unroll
+          for (int kk = 0; kk < kHD / 16; ++kk)
+            mma_bf16(tmem + kTcKeys * st, sdesc(sQ + kk * 32), sdesc(kb + kk * 32), idesc_s, kk > 0 ? 1u : 0u);
+          mma_commit(smem_u32(&s_full[st]));
+          if (j == r.n - 1) mma_commit(smem_u32(q_empty));
+          if (pv >= 0 && !issue_pv(pv, pv_first)) { ok = false; break; }
+          pv = g;
+          pv_first = j == 0;
+          // the item's last P V follows at once: the softmax's read of O
+          // does not wait for the next item's copies
+          if (j == r.n - 1) {
+            if (!issue_pv(pv, pv_first)) { ok = false; break; }
+            pv = -1;
+          }
+        }
+        if (ok && r.n == 0) mma_commit(smem_u32(q_empty));
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
     }
+    if (lane == 0 && ok && pv >= 0) issue_pv(pv, pv_first);
     __syncwarp();
   } else {
     // softmax: kTcSplit threads per query row, `part` of its keys and output each
@@ -507,129 +604,140 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     const float sc = 1.4426950408889634f * rsqrtf((float)kHD);
     const uint32_t lane_base = (uint32_t)(32 * quarter) << 16;
     const int kb0 = kTcPart * part;               // first key of this thread's part of a tile
-    // m: the row max the probabilities of the tiles so far are taken
-    // against (raised only when a tile's max exceeds it by more than 2^8, so
-    // P stays below 256); l: this thread's part of their sum
     constexpr float kRescale = 8.f;
-    float m = -INFINITY, l = 0.f;
     // this row's 16-byte chunks of P buffer 0 for keys kb0 .. kb0 + 31: atom
     // kb0 / 64, chunks (kb0 % 64) / 8 + q at position chunk ^ (row % 8)
     const uint32_t prow = sP + (kb0 >> 6) * (kTcP / 2) + row * 128;
     const int chunk0 = (kb0 & 63) >> 3;
-    bool ok = true;
-    // the visible keys kb0 + i (i < kTcPart) of a row as a bit mask: [lo, hi) relative to the tile
-    auto range_bits = [&](int lo, int hi) -> unsigned long long {
-      lo = max(lo - kb0, 0);
-      hi = min(hi - kb0, kTcPart);
-      if (hi <= lo) return 0ull;
-      const unsigned long long up = hi >= 64 ? ~0ull : ((1ull << hi) - 1ull);
-      return up & ~((1ull << lo) - 1ull);
-    };
-    // A bounded wait that runs out raises s_abort; every softmax thread reads
-    // it after the next barrier, so all of them leave the loop together.
-    auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) {
-      if (!mbar_wait(smem_u32(bar), parity, d_err)) *s_abort = 1;
-    };
     // this thread's output dims of the O accumulator in TMEM
     const uint32_t o_addr = tmem + lane_base + 256 + kTcOut * part;
-    for (int j = 0; j < n_tiles; ++j) {
-      const int st = j & 1;
-      int kt, kend;
-      tile_at(j, &kt, &kend);
-      // visible keys of this part: the context prefix [0, ctx], the windows,
-      // none past the range's end (each key belongs to one range's tiles)
-      const int lim = min(kend - kt, kTcKeys);
-      const bool open = !a.dense && kt + kTcKeys - 1 < kend && kt + kTcKeys - 1 <= cmin && v.ctx >= 0;
-      unsigned long long vis = ~0ull;
-      if (!open)
-        vis = (range_bits(0, v.ctx - kt + 1) | range_bits(v.w1lo - kt, v.w1hi - kt) |
-               range_bits(v.w2lo - kt, v.w2hi - kt)) &
-              range_bits(0, lim);
-      wait_or_abort(&s_full[st], (j >> 1) & 1);
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      float sv[kTcPart];
-#pragma unroll
-      for (int c = 0; c < kTcPart / 32; ++c) tmem_ld32(tmem + lane_base + kTcKeys * st + kb0 + 32 * c, sv + 32 * c);
-      // raw scores: sc > 0, so the max commutes with the scaling
-      float mx = -INFINITY;
-#pragma unroll
-      for (int e = 0; e < kTcPart; ++e) {
-        sv[e] = ((vis >> e) & 1ull) ? sv[e] : -INFINITY;
-        mx = fmaxf(mx, sv[e]);
-      }
-      // the row's max over its parts
-      s_mx[(st * kTcSplit + part) * kTcRows + row] = mx;
-      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
-      if (*s_abort) { ok = false; break; }
-      mx = s_mx[(st * kTcSplit) * kTcRows + row];
-#pragma unroll
-      for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
-      // A new reference max when this tile's exceeds it by more than 2^8: O
-      // and l so far are scaled to it (O once the previous tile's P V has
-      // landed; nothing is accumulated before a finite max).  The TMEM
-      // load and store are warp-wide: a warp rescales when any of its rows
-      // needs it, the others by 1.
-      const bool raise = mx * sc > m + kRescale;
-      const float f = (raise && m != -INFINITY) ? ex2(m - mx * sc) : 1.f;
-      if (__any_sync(0xffffffffu, f != 1.f)) {
-        wait_or_abort(&o_full[(j - 1) & 1], ((j - 1) >> 1) & 1);
+    // A bounded wait that runs out marks the thread failed; the next
+    // OR-barrier tells every softmax thread, and all leave the loops.
+    bool failed = false;
+    auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) {
+      if (!mbar_wait(smem_u32(bar), parity, d_err)) failed = true;
+    };
+    bool ok = true;
+    int g = 0, it = 0;
+    for (int w = item_at(0); ok && w >= 0; w = item_at(++it)) {
+      int q0, h, b;
+      item(w, &q0, &h, &b);
+      const TileRanges r = tile_ranges(a, q0, lane);
+      const RowVis v = row_vis(a, q0 + row);
+      // the visible keys kb0 + i (i < kTcPart) of a row as a bit mask: [lo, hi) relative to the tile
+      auto range_bits = [&](int lo, int hi) -> unsigned long long {
+        lo = max(lo - kb0, 0);
+        hi = min(hi - kb0, kTcPart);
+        if (hi <= lo) return 0ull;
+        const unsigned long long up = hi >= 64 ? ~0ull : ((1ull << hi) - 1ull);
+        return up & ~((1ull << lo) - 1ull);
+      };
+      // m: the row max the probabilities of the item's tiles so far are
+      // taken against (raised only when a tile's max exceeds it by more than
+      // 2^8, so P stays below 256); l: this thread's part of their sum
+      float m = -INFINITY, l = 0.f;
+      for (int j = 0; j < r.n; ++j, ++g) {
+        const int st = g & 1;
+        int kt, kend;
+        tile_at(r, j, &kt, &kend);
+        // visible keys of this part: the context prefix [0, ctx], the windows,
+        // none past the range's end (each key belongs to one range's tiles)
+        const int lim = min(kend - kt, kTcKeys);
+        const bool open = !a.dense && kt + kTcKeys - 1 < kend && kt + kTcKeys - 1 <= r.cmin && v.ctx >= 0;
+        unsigned long long vis = ~0ull;
+        if (!open)
+          vis = (range_bits(0, v.ctx - kt + 1) | range_bits(v.w1lo - kt, v.w1hi - kt) |
+                 range_bits(v.w2lo - kt, v.w2hi - kt)) &
+                range_bits(0, lim);
+        wait_or_abort(&s_full[st], (g >> 1) & 1);
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        float r[kTcOut];
-        tmem_ld32(o_addr, r);
+        float sv[kTcPart];
 #pragma unroll
-        for (int d = 0; d < kTcOut; ++d) r[d] *= f;
-        tmem_st32(o_addr, r);
-      }
-      if (raise) {
-        l *= f;
-        m = mx * sc;
-      }
-      const float mn = m;
-      // P = exp2(S sc - mn) rounded to bf16 (ex2(-inf) = 0 for masked keys),
-      // the sum of the rounded values
-      const uint32_t pbase = prow + st * kTcP;
-      const float nmn = mn == -INFINITY ? 0.f : -mn;
-      float ps = 0.f;
+        for (int c = 0; c < kTcPart / 32; ++c) tmem_ld32(tmem + lane_base + kTcKeys * st + kb0 + 32 * c, sv + 32 * c);
+        // raw scores: sc > 0, so the max commutes with the scaling
+        float mx = -INFINITY;
 #pragma unroll
-      for (int q = 0; q < kTcPart / 8; ++q) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int e = 8 * q + 2 * u;
-          pk[u] = pack_bf16(ex2(fmaf(sv[e], sc, nmn)), ex2(fmaf(sv[e + 1], sc, nmn)));
-          const float2 f = unpack_bf16(pk[u]);
-          ps += f.x + f.y;
+        for (int e = 0; e < kTcPart; ++e) {
+          sv[e] = ((vis >> e) & 1ull) ? sv[e] : -INFINITY;
+          mx = fmaxf(mx, sv[e]);
         }
-        const uint32_t addr = pbase + (((chunk0 + q) ^ (row & 7)) << 4);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
-                     "r"(pk[3])
-                     : "memory");
-      }
-      l += ps;
-      // S_j read, P_j written: to the tensor cores (async proxy)
-      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
-      if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
-    }
-    float o[kTcOut];
+        // the row's max over its parts
+        s_mx[(st * kTcSplit + part) * kTcRows + row] = mx;
+        if (softmax_bar_or(failed)) { ok = false; break; }
+        mx = s_mx[(st * kTcSplit) * kTcRows + row];
 #pragma unroll
-    for (int d = 0; d < kTcOut; ++d) o[d] = 0.f;
-    if (ok && n_tiles > 0) {
-      // the last tile's P V completes the accumulator
-      wait_or_abort(&o_full[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1);
-      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      tmem_ld32(o_addr, o);
-      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
-      if (*s_abort) ok = false;
-    }
-    if (ok) {
-      // the row's sum over its parts, in a fixed order
-      s_l[part * kTcRows + row] = l;
+        for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
+        // A new reference max when this tile's exceeds it by more than 2^8: O
+        // and l so far are scaled to it (O once the previous tile's P V has
+        // landed; nothing is accumulated before a finite max).  The TMEM
+        // load and store are warp-wide: a warp rescales when any of its rows
+        // needs it, the others by 1.
+        const bool raise = mx * sc > m + kRescale;
+        const float f = (raise && m != -INFINITY) ? ex2(m - mx * sc) : 1.f;
+        if (__any_sync(0xffffffffu, f != 1.f)) {
+          wait_or_abort(&o_full[(g - 1) & 1], ((g - 1) >> 1) & 1);
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          float rr[kTcOut];
+          tmem_ld32(o_addr, rr);
+#pragma unroll
+          for (int d = 0; d < kTcOut; ++d) rr[d] *= f;
+          tmem_st32(o_addr, rr);
+        }
+        if (raise) {
+          l *= f;
+          m = mx * sc;
+        }
+        const float mn = m;
+        // P = exp2(S sc - mn) rounded to bf16 (ex2(-inf) = 0 for masked keys),
+        // the sum of the rounded values
+        const uint32_t pbase = prow + st * kTcP;
+        const float nmn = mn == -INFINITY ? 0.f : -mn;
+        float ps = 0.f;
+#pragma unroll
+        for (int q = 0; q < kTcPart / 8; ++q) {
+          uint32_t pk[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int e = 8 * q + 2 * u;
+            pk[u] = pack_bf16(ex2(fmaf(sv[e], sc, nmn)), ex2(fmaf(sv[e + 1], sc, nmn)));
+            const float2 pf = unpack_bf16(pk[u]);
+            ps += pf.x + pf.y;
+          }
+          const uint32_t addr = pbase + (((chunk0 + q) ^ (row & 7)) << 4);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
+                       "r"(pk[3])
+                       : "memory");
+        }
+        l += ps;
+        // S_g read, P_g written: to the tensor cores (async proxy)
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+        if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
+      }
+      if (!ok) break;
+      float o[kTcOut];
+#pragma unroll
+      for (int d = 0; d < kTcOut; ++d) o[d] = 0.f;
+      if (r.n > 0) {
+        // the item's last P V completes the accumulator; once every softmax
+        // thread has read it, the next item's first P V may overwrite it
+        wait_or_abort(&o_full[(g - 1) & 1], ((g - 1) >> 1) & 1);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        tmem_ld32(o_addr, o);
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        if (softmax_bar_or(failed)) { ok = false; break; }
+        if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(o_free)) : "memory");
+      }
+      // the row's sum over its parts, in a fixed order (one buffer per item
+      // parity: a thread writes the next item's sums only after the barrier
+      // below, which every thread passes after reading this item's)
+      float* sl = s_l + (it & 1) * kTcSplit * kTcRows;
+      sl[part * kTcRows + row] = l;
       asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
       float lt = 0.f;
 #pragma unroll
-      for (int q = 0; q < kTcSplit; ++q) lt += s_l[q * kTcRows + row];
+      for (int q = 0; q < kTcSplit; ++q) lt += sl[q * kTcRows + row];
       const int qi = q0 + row;
       if (qi < a.q_end && lt > 0.f) {
         const float inv = 1.f / lt;
@@ -687,7 +795,10 @@ extern "C" int kf_op_train_attention(int32_t blocks, int32_t B, int32_t H, int32
   if (!err) return KF_E_CUDA;
   static PerDevice attr_tc;
   set_smem_attr(attr_tc, k_train_attention_tc, tc_smem_bytes());
-  const dim3 grid(ceil_div(q_end - q_begin, kTcRows), H, B);
-  kf_launch(k_train_attention_tc, grid, dim3(kTcThreads), tc_smem_bytes(), s, mq, mk, mv, a, err);
+  // persistent: one CTA per SM over the (query tile, head, sequence) items
+  const long long items = (long long)ceil_div(q_end - q_begin, kTcRows) * H * B;
+  if (items > (1ll << 30)) return KF_E_ARG;
+  const dim3 grid((unsigned)std::min<long long>(items, device_sms()));
+  kf_launch(k_train_attention_tc, grid, dim3(kTcThreads), tc_smem_bytes(), s, mq, mk, mv, a, (int)B, err);
   return cudaGetLastError() == cudaSuccess ? KF_OK : KF_E_CUDA;
 }

@@ -118,3 +118,21 @@ def test_argument_errors(env):
         assert lib.kf_op_train_attention(*args, p, p, p, out.data_ptr(), 0, None) == -1, args
     # an unknown flag
     assert lib.kf_op_train_attention(1, 1, 1, 4, 2, 0, 12, p, p, p, out.data_ptr(), 4, None) == -1
+
+
+@pytest.mark.parametrize("blocks,B,H,N,k", [(1, 4, 12, 128, 4), (1, 4, 12, 256, 4), (2, 2, 12, 256, 4)])
+def test_many_items_per_cta(env, blocks, B, H, N, k):
+    """More (query tile, head, sequence) items than SMs, so each persistent
+    CTA carries its tiles, buffers and row sums across several items: every
+    row against the warp-level MMA kernel, sampled rows against the oracle."""
+    torch, lib = env
+    T = N + blocks * N * k
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, dense=0, seed=N + B)
+    out2 = _run(torch, lib, blocks, B, H, N, k, dense=2, seed=N + B)[3]
+    assert np.isfinite(out).all()
+    assert np.abs(out - out2).max() <= 8e-3 * np.abs(v).max()
+    mask = ta.mask_full(N, k, blocks)
+    rows = np.array([0, 127, N - 1, N, N + 5, N + N * k // 2 + 1, N + N * k - 1, T - 1])
+    for b in range(B):
+        ref = ta.masked_attention(q[b, rows], kk[b], v[b], mask[rows])
+        assert np.abs(out[b, rows] - ref).max() <= 8e-3 * np.abs(v[b]).max()
