@@ -308,10 +308,13 @@ __global__ void __launch_bounds__(kThr, 3) k_train_attention(TrainAttnArgs a) {
 //   warps 2..9  two threads per query row (TMEM lane), each with half of
 //               its keys and of its output (four threads measured 5 % slower:
 //               the per-tile chain of waits and barriers, not the arithmetic,
-//               bounds the softmax): mask S_j, share the row max
-//               through shared memory, keep a reference max m and their
-//               part of the sum l, and write P_j = exp2(S_j - m) as bf16 into
-//               shared memory (K-major, swizzled: the A operand of P V).  m
+//               bounds the softmax): mask S_j, share the row max with the
+//               partner warp (the other half of the same rows) through shared
+//               memory and a barrier of the pair, keep a reference max m and
+//               their part of the sum l, and write P_j = exp2(S_j - m) as
+//               bf16 into shared memory (K-major, swizzled: the A operand of
+//               P V); every softmax thread arrives on the barrier that
+//               releases P_j to the tensor cores.  m
 //               is raised only when a tile's max exceeds it by more than 2^8
 //               (P stays below 256); then O in TMEM and l are scaled to the
 //               new m before P_j is released.  At the item's end O / l is
@@ -384,19 +387,50 @@ __device__ __forceinline__ TileRanges tile_ranges(const TrainAttnArgs& a, int q0
   return r;
 }
 
-// named barrier 1 over the softmax threads that also ORs a predicate over
-// them: every thread gets the same answer, so all leave a loop together
-__device__ __forceinline__ bool softmax_bar_or(bool pred) {
+// The two softmax warps of a TMEM lane quarter hold the two parts of the same
+// rows; they meet on named barrier 2 + quarter (64 threads), which also ORs
+// a predicate over them: both get the same answer and leave a loop together.
+__device__ __forceinline__ bool pair_bar_or(int quarter, bool pred) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred p, q;\n\t"
       "setp.ne.u32 p, %1, 0;\n\t"
-      "bar.red.or.pred q, 1, %2, p;\n\t"
+      "bar.red.or.pred q, %2, 64, p;\n\t"
       "selp.u32 %0, 1, 0, q;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)pred), "n"(kTcSoftmax)
+      : "r"((uint32_t)pred), "r"(2 + quarter)
       : "memory");
   return r != 0;
+}
+__device__ __forceinline__ void pair_bar(int quarter) {
+  asm volatile("bar.sync %0, 64;" ::"r"(2 + quarter) : "memory");
+}
+
+// three-way max, and packed pairs of fp32 (two lanes of one 64-bit register)
+__device__ __forceinline__ float max3f(float x, float y, float z) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(x), "f"(y), "f"(z));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2(float x, float y) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+  return r;
+}
+__device__ __forceinline__ float2 f2_split(uint64_t p) {
+  float2 r;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(p));
+  return r;
+}
+__device__ __forceinline__ uint64_t fma_f2(uint64_t x, uint64_t y, uint64_t z) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(x), "l"(y), "l"(z));
+  return r;
+}
+__device__ __forceinline__ uint64_t add_f2(uint64_t x, uint64_t y) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(x), "l"(y));
+  return r;
 }
 
 // first key and range end of tile j of an item (constant indices only: the
@@ -471,10 +505,10 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&s_full[i]), 1);
-      mbar_init(smem_u32(&p_full[i]), 1);
+      mbar_init(smem_u32(&p_full[i]), kTcSoftmax);      // every softmax thread
       mbar_init(smem_u32(&o_full[i]), 1);
     }
-    mbar_init(smem_u32(o_free), 1);
+    mbar_init(smem_u32(o_free), kTcSoftmax);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_q)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_k)) : "memory");
@@ -612,7 +646,8 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
     // this thread's output dims of the O accumulator in TMEM
     const uint32_t o_addr = tmem + lane_base + 256 + kTcOut * part;
     // A bounded wait that runs out marks the thread failed; the next
-    // OR-barrier tells every softmax thread, and all leave the loops.
+    // OR-barrier tells its partner warp, and both leave the loops (the other
+    // pairs' waits then run out in turn).
     bool failed = false;
     auto wait_or_abort = [&](uint64_t* bar, uint32_t parity) {
       if (!mbar_wait(smem_u32(bar), parity, d_err)) failed = true;
@@ -655,15 +690,20 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
 #pragma unroll
         for (int c = 0; c < kTcPart / 32; ++c) tmem_ld32(tmem + lane_base + kTcKeys * st + kb0 + 32 * c, sv + 32 * c);
         // raw scores: sc > 0, so the max commutes with the scaling
-        float mx = -INFINITY;
+        if (vis != ~0ull) {
 #pragma unroll
-        for (int e = 0; e < kTcPart; ++e) {
-          sv[e] = ((vis >> e) & 1ull) ? sv[e] : -INFINITY;
-          mx = fmaxf(mx, sv[e]);
+          for (int e = 0; e < kTcPart; ++e) sv[e] = ((vis >> e) & 1ull) ? sv[e] : -INFINITY;
         }
-        // the row's max over its parts
+        // four independent max chains, then combined
+        float mq[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int e = 0; e < kTcPart; e += 8)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) mq[c] = max3f(mq[c], sv[e + 2 * c], sv[e + 2 * c + 1]);
+        float mx = fmaxf(fmaxf(mq[0], mq[1]), fmaxf(mq[2], mq[3]));
+        // the row's max over its parts (the partner warp)
         s_mx[(st * kTcSplit + part) * kTcRows + row] = mx;
-        if (softmax_bar_or(failed)) { ok = false; break; }
+        if (pair_bar_or(quarter, failed)) { ok = false; break; }
         mx = s_mx[(st * kTcSplit) * kTcRows + row];
 #pragma unroll
         for (int q = 1; q < kTcSplit; ++q) mx = fmaxf(mx, s_mx[(st * kTcSplit + q) * kTcRows + row]);
@@ -692,28 +732,31 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
         // the sum of the rounded values
         const uint32_t pbase = prow + st * kTcP;
         const float nmn = mn == -INFINITY ? 0.f : -mn;
-        float ps = 0.f;
+        const uint64_t sc2 = f2(sc, sc), nmn2 = f2(nmn, nmn);
+        uint64_t ps2[4] = {f2(0.f, 0.f), f2(0.f, 0.f), f2(0.f, 0.f), f2(0.f, 0.f)};   // independent sums
 #pragma unroll
         for (int q = 0; q < kTcPart / 8; ++q) {
           uint32_t pk[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const int e = 8 * q + 2 * u;
-            pk[u] = pack_bf16(ex2(fmaf(sv[e], sc, nmn)), ex2(fmaf(sv[e + 1], sc, nmn)));
+            const float2 arg = f2_split(fma_f2(f2(sv[e], sv[e + 1]), sc2, nmn2));
+            pk[u] = pack_bf16(ex2(arg.x), ex2(arg.y));
             const float2 pf = unpack_bf16(pk[u]);
-            ps += pf.x + pf.y;
+            ps2[u] = add_f2(ps2[u], f2(pf.x, pf.y));
           }
           const uint32_t addr = pbase + (((chunk0 + q) ^ (row & 7)) << 4);
           asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(pk[0]), "r"(pk[1]), "r"(pk[2]),
                        "r"(pk[3])
                        : "memory");
         }
-        l += ps;
-        // S_g read, P_g written: to the tensor cores (async proxy)
+        const float2 ps = f2_split(add_f2(add_f2(ps2[0], ps2[1]), add_f2(ps2[2], ps2[3])));
+        l += ps.x + ps.y;
+        // S_g read, P_g written: to the tensor cores (async proxy); every
+        // softmax thread arrives
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
-        if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
+        asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&p_full[st])) : "memory");
       }
       if (!ok) break;
       float o[kTcOut];
@@ -726,15 +769,15 @@ k_train_attention_tc(const __grid_constant__ CUtensorMap map_q, const __grid_con
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         tmem_ld32(o_addr, o);
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        if (softmax_bar_or(failed)) { ok = false; break; }
-        if (t == 64) asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(o_free)) : "memory");
+        if (pair_bar_or(quarter, failed)) { ok = false; break; }
+        asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(o_free)) : "memory");
       }
       // the row's sum over its parts, in a fixed order (one buffer per item
-      // parity: a thread writes the next item's sums only after the barrier
-      // below, which every thread passes after reading this item's)
+      // parity: a thread writes the next item's sums only after the pair
+      // barrier below, which its partner passes after reading this item's)
       float* sl = s_l + (it & 1) * kTcSplit * kTcRows;
       sl[part * kTcRows + row] = l;
-      asm volatile("bar.sync 1, %0;" ::"n"(kTcSoftmax) : "memory");
+      pair_bar(quarter);
       float lt = 0.f;
 #pragma unroll
       for (int q = 0; q < kTcSplit; ++q) lt += sl[q * kTcRows + row];
