@@ -136,3 +136,21 @@ def test_many_items_per_cta(env, blocks, B, H, N, k):
     for b in range(B):
         ref = ta.masked_attention(q[b, rows], kk[b], v[b], mask[rows])
         assert np.abs(out[b, rows] - ref).max() <= 8e-3 * np.abs(v[b]).max()
+
+
+def test_future2_rows_many_items(env):
+    """DoubleForward's Future-2 rows only (q_begin > 0) over more items than
+    SMs: every row against the warp-level MMA kernel, sampled rows against
+    the oracle."""
+    torch, lib = env
+    blocks, B, H, N, k = 2, 2, 12, 256, 4
+    qb, qe = N + N * k, N + 2 * N * k
+    q, kk, v, out = _run(torch, lib, blocks, B, H, N, k, qb, qe, seed=13)
+    out2 = _run(torch, lib, blocks, B, H, N, k, qb, qe, dense=2, seed=13)[3]
+    assert np.isfinite(out).all()
+    assert np.abs(out - out2).max() <= 8e-3 * np.abs(v).max()
+    mask = ta.mask_full(N, k, blocks)[qb:qe]
+    rel = np.array([0, 1, 127, 128, 511, 777, qe - qb - 1])
+    for b in range(B):
+        ref = ta.masked_attention(q[b, qb + rel], kk[b], v[b], mask[rel])
+        assert np.abs(out[b, rel] - ref).max() <= 8e-3 * np.abs(v[b]).max()
